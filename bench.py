@@ -1,0 +1,417 @@
+#!/usr/bin/env python
+"""Benchmark: one SPSA step of the shared-randomness method on OPT-shaped
+synthetic parameters, through the C ABI of libjb.
+
+A step is one pass of the whole hot path over the parameter set:
+  perturb(+eps), perturb(-2 eps), perturb(+eps)  one SPSA sample around its two
+                                                 loss evaluations (Algorithm 1)
+  quantize the sample's projected gradient       one byte (Section 3)
+  fused update of K machines' (seed, byte) pairs (Section 2; Algorithm 1)
+The loss evaluations themselves (model forwards) are outside the path; the
+projected gradient is a seeded synthetic scalar.
+
+Metric: param.seed updates/s = N (K + 3) / step time, the whole job over all
+ranks. Inputs (25.7 GB for the 13B-shaped set) are far larger than L2, so no
+flush is needed between steps. Ranks (torchrun, N > 1) are independent
+replicas: the path has no exchange step on the device.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl jb|reference]
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "param·seed updates/s and HBM GB/s (% roofline), 13B-shaped bf16, K=64"
+UNIT = "param·seed/s"
+
+# Algorithmic lane operations per element-seed (the ALU roofline's unit of work):
+# a quarter Philox4x32-10 block (10 rounds x 2 wide multiplies + 2 three-way XORs,
+# over 4 words) = 10; half a Box-Muller pair (2 uniform conversions, log, sqrt,
+# sin, cos, 2 products over 2 elements) = 4; the accumulate FMA = 1.
+OPS_PER_PARAM_SEED = 15
+LANES_PER_SM_CLK = 128
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=5)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=["jb", "reference"], default="jb")
+    ap.add_argument("--model", default="opt-13b")
+    ap.add_argument("--dtype", choices=["bf16", "f32"], default="bf16")
+    ap.add_argument("--K", type=int, default=64)
+    ap.add_argument("--eps", type=float, default=1e-3)
+    ap.add_argument("--lr", type=float, default=1e-6)
+    ap.add_argument("--qscale", type=float, default=16.0)
+    ap.add_argument("--e2e-steps", type=int, default=2)
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=12.0,
+                    help="target CPU time of the oracle sample")
+    ap.add_argument("--sweep", default="", help="comma list of K: time update/perturb per K")
+    ap.add_argument("--sweep-out", default="", help="file for the sweep's JSON lines")
+    return ap.parse_args()
+
+
+def dist_env():
+    return (int(os.environ.get("RANK", 0)), int(os.environ.get("LOCAL_RANK", 0)),
+            int(os.environ.get("WORLD_SIZE", 1)))
+
+
+def workload_name(a) -> str:
+    return f"{a.model}-shaped {a.dtype}, SPSA step (perturb +eps/-2eps/+eps, K={a.K} fused update)"
+
+
+# --- clocks ------------------------------------------------------------------------
+
+class ClockSampler:
+    FIELDS = ["clocks.sm", "clocks.max.sm", "power.draw", "clocks_event_reasons.hw_slowdown",
+              "clocks_event_reasons.hw_thermal_slowdown", "clocks_event_reasons.sw_thermal_slowdown",
+              "clocks_event_reasons.sw_power_cap"]
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+        self.lines = []
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), "--query-gpu=" + ",".join(self.FIELDS),
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.thread = threading.Thread(target=self._read, daemon=True)
+            self.thread.start()
+        except OSError:
+            self.proc = None
+
+    def _read(self):
+        for ln in self.proc.stdout:
+            self.lines.append(ln.strip())
+
+    def stop(self) -> dict:
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.thread.join(timeout=5)
+        sm, smax, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            parts = [p.strip() for p in ln.split(",")]
+            if len(parts) != len(self.FIELDS):
+                continue
+            try:
+                sm.append(float(parts[0]))
+                smax.append(float(parts[1]))
+            except ValueError:
+                continue
+            for name, v in zip(names, parts[3:]):
+                if v.lower().startswith("active"):
+                    reasons.add(name)
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(smax) if smax else None, "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# --- the CPU oracle (baseline and reference arm) --------------------------------------
+
+def oracle_rate(a, target_s: float):
+    """The oracle, as it stands, on a bounded sample of the workload: sampled
+    elements x (3 perturb seeds + K update seeds). Returns (param.seed/s, cores, sample)."""
+    import numpy as np
+
+    import oracle
+    import synthetic
+    cores = len(os.sched_getaffinity(0))
+    oracle.set_threads(cores)
+    specs = synthetic.opt_tensors(a.model)
+    numels = [s.numel for s in specs]
+    offs = synthetic.flat_offsets(numels)
+    seeds = [(int(m), 0, 0) for m in synthetic.machine_ids(a.K, 900)]
+    q = synthetic.byte_codes(a.K, 900, 0)
+    own = seeds[0]
+
+    def run(n):
+        pos = synthetic.sample_positions(numels, n, 901)
+        idx = np.concatenate([fo + p for fo, p in zip(offs, pos)]).astype(np.uint64)
+        vals = synthetic.normal_values(idx.size, 0.02, 902)
+        if a.dtype == "bf16":
+            vals = oracle.round_bf16(vals.astype(np.float64)) if idx.size < 4096 else \
+                (vals.view(np.uint32) >> 16).astype(np.uint16)
+        t0 = time.perf_counter()
+        v = vals
+        for e in (a.eps, -2 * a.eps, a.eps):
+            v = oracle.perturb_at(v, idx, own, e)
+        oracle.update_at(v, idx, seeds, q, a.lr, 1.0, a.qscale)
+        return idx.size, time.perf_counter() - t0
+
+    n0, t0 = run(1 << 12)
+    rate = n0 * (a.K + 3) / max(t0, 1e-6)
+    n = int(min(max(rate * target_s / (a.K + 3), 1 << 12), 1 << 26))
+    n, t = run(n)
+    return n * (a.K + 3) / t, cores, t, n
+
+
+def run_reference(a):
+    rank, _, world = dist_env()
+    if rank != 0:
+        return
+    steps_rates = []
+    n_used = 0
+    cores = 0
+    for _ in range(max(a.steps, 1)):
+        rate, cores, t, n_used = oracle_rate(a, min(a.cpu_seconds, 60.0 / max(a.steps, 1)))
+        steps_rates.append(rate)
+    value = statistics.median(steps_rates)
+    sample = (f"{n_used} sampled elements of the {a.model}-shaped set per step, each taking "
+              f"3 perturb seeds and {a.K} update seeds")
+    print(json.dumps({
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": a.gpus,
+        "steps": a.steps, "warmup": a.warmup, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": workload_name(a), "K": a.K},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
+                         "sample": sample},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }), flush=True)
+
+
+# --- the GPU arm -----------------------------------------------------------------------
+
+def main():
+    a = parse()
+    if a.impl == "reference":
+        run_reference(a)
+        return
+    import numpy as np
+    import torch
+
+    import paper_2306_10015_gb300 as jb
+    import synthetic
+
+    rank, local_rank, world = dist_env()
+    torch.cuda.set_device(local_rank)
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local_rank))
+    else:
+        dist = None
+
+    def barrier():
+        if dist is not None:
+            dist.barrier()
+
+    tdt = torch.bfloat16 if a.dtype == "bf16" else torch.float32
+    esize = 2 if a.dtype == "bf16" else 4
+    specs, tensors, offs = synthetic.opt_parameters(a.model, tdt, seed=synthetic.MASTER_SEED + rank)
+    table = jb.ParamTable(tensors, offs)
+    N = table.numel
+    K = a.K
+    mids = synthetic.machine_ids(K, 900)
+    own = 0  # this replica's machine is the first of the K
+    n_total = a.warmup + a.steps + a.e2e_steps + 1
+    seeds = [jb.seeds_array([(int(m), t, 0) for m in mids]) for t in range(n_total)]
+    codes = [synthetic.byte_codes(K, 900, t) for t in range(n_total)]
+    ghat = synthetic.rng(903).standard_normal(n_total) * 100.0
+    stream = torch.cuda.current_stream()
+    launches_per_step = 3 * (-(-table.n_segments // 1000)) + (-(-table.n_segments // 700))
+
+    ev = {}
+
+    def step(t, timed=False):
+        s_own = (int(mids[own]), t, 0)
+        if timed:
+            ev.setdefault("p0", []).append(torch.cuda.Event(enable_timing=True))
+            ev["p0"][-1].record(stream)
+        jb.jb_perturb(table, s_own, a.eps, stream)
+        jb.jb_perturb(table, s_own, -2 * a.eps, stream)
+        jb.jb_perturb(table, s_own, a.eps, stream)
+        q = codes[t]
+        q[own] = jb.jb_quantize_grad(float(ghat[t]), a.qscale)
+        if timed:
+            ev.setdefault("u0", []).append(torch.cuda.Event(enable_timing=True))
+            ev["u0"][-1].record(stream)
+        jb.jb_apply_updates(table, seeds[t], q, a.lr, 1.0, a.qscale, stream)
+        if timed:
+            ev.setdefault("u1", []).append(torch.cuda.Event(enable_timing=True))
+            ev["u1"][-1].record(stream)
+
+    for t in range(a.warmup):
+        step(t)
+    torch.cuda.synchronize()
+    barrier()
+    torch.cuda.synchronize()
+    clocks = ClockSampler(local_rank)
+    clocks.start()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for t in range(a.warmup, a.warmup + a.steps):
+        step(t, timed=True)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    barrier()
+    clk = clocks.stop()
+    ms = e0.elapsed_time(e1)
+    upd_ms = [x.elapsed_time(y) for x, y in zip(ev["u0"], ev["u1"])]
+    pert_ms = [x.elapsed_time(y) / 3 for x, y in zip(ev["p0"], ev["u0"])]
+    if dist is not None:
+        tt = torch.tensor([ms], device="cuda")
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        ms = float(tt.item())
+    ms_per_step = ms / a.steps
+    units_per_step = N * (K + 3) * world
+    value = units_per_step / (ms_per_step / 1e3)
+
+    # end to end through the same public calls, theta in pinned host memory
+    e2e = None
+    if not a.no_e2e:
+        host = [torch.empty(t.shape, dtype=t.dtype, pin_memory=True) for t in tensors]
+        for h, d in zip(host, tensors):
+            h.copy_(d)
+        torch.cuda.synchronize()
+
+        def e2e_step(t):
+            for h, d in zip(host, tensors):
+                d.copy_(h, non_blocking=True)
+            step(t)
+            for h, d in zip(host, tensors):
+                h.copy_(d, non_blocking=True)
+        base = a.warmup + a.steps
+        e2e_step(base)
+        torch.cuda.synchronize()
+        barrier()
+        x0, x1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        x0.record(stream)
+        for t in range(base + 1, base + 1 + a.e2e_steps):
+            e2e_step(t)
+        x1.record(stream)
+        torch.cuda.synchronize()
+        xms = x0.elapsed_time(x1) / a.e2e_steps
+        if dist is not None:
+            tt = torch.tensor([xms], device="cuda")
+            dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+            xms = float(tt.item())
+        e2e = {"value": units_per_step / (xms / 1e3), "unit": UNIT,
+               "h2d_bytes_per_step": N * esize, "d2h_bytes_per_step": N * esize,
+               "ms_per_step": xms}
+        del host
+
+    sweep_lines = []
+    if a.sweep and rank == 0:
+        sweep_lines = run_sweep(a, jb, table, mids, stream)
+
+    if rank != 0:
+        if dist is not None:
+            dist.destroy_process_group()
+        return
+
+    props = torch.cuda.get_device_properties(local_rank)
+    sms = props.multi_processor_count
+    peaks = {}
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            peaks = json.load(f)
+    except OSError:
+        pass
+    hbm_peak = float(peaks.get("hbm_gbs", 6800.0))
+    f_max = float(peaks.get("sm_max_mhz", 2070.0)) * 1e6
+    upd = statistics.mean(upd_ms) / 1e3
+    alu_peak = sms * LANES_PER_SM_CLK * f_max / 1e12            # Tops/s
+    alu_ach = OPS_PER_PARAM_SEED * K * N / upd / 1e12
+    traffic = load_traffic(a)
+    roofline = {"bound": "alu", "achieved": alu_ach, "peak": alu_peak, "unit": "Tops/s",
+                "frac": alu_ach / alu_peak, "traffic": traffic,
+                "kernel": "seeded_kernel<bf16, update>" if a.dtype == "bf16" else
+                "seeded_kernel<f32, update>",
+                "ops_per_param_seed": OPS_PER_PARAM_SEED,
+                "peak_basis": f"{sms} SMs x {LANES_PER_SM_CLK} lanes x {f_max / 1e6:.0f} MHz",
+                "hbm_gbs": 2 * esize * N / upd / 1e9, "hbm_frac_of_measured": 2 * esize * N / upd / 1e9 / hbm_peak,
+                "update_ms": statistics.mean(upd_ms), "perturb_ms": statistics.mean(pert_ms)}
+    cpu = None
+    if not a.no_cpu_baseline and world == 1:
+        rate, cores, t, n = oracle_rate(a, a.cpu_seconds)
+        cpu = {"value": rate, "unit": UNIT, "cores": cores, "kind": "oracle",
+               "sample": f"{n} sampled elements x (3 perturb + {K} update seeds), {t:.1f} s"}
+    step_bytes = 4 * 2 * esize * N  # 3 perturb passes + 1 update pass, read + write
+    out = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": a.steps,
+        "warmup": a.warmup, "ms_per_step": ms_per_step, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": a.dtype, "data": "synthetic",
+        "config": {"workload": workload_name(a), "n_params": N, "n_tensors": table.n_segments,
+                   "K": K, "eps": a.eps, "lr": a.lr, "qscale": a.qscale,
+                   "l2": "inputs larger than L2 (no flush needed)",
+                   "parallelism": f"replicas x{world}"},
+        "hbm_gbs_step": step_bytes * world / (ms_per_step / 1e3) / 1e9,
+        "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e,
+        "gpu_launches": launches_per_step * a.steps, "clocks": clk,
+    }
+    if sweep_lines:
+        out["sweep"] = sweep_lines
+    print(json.dumps(out), flush=True)
+    if dist is not None:
+        dist.destroy_process_group()
+
+
+def load_traffic(a):
+    """dram bytes per update launch from a committed ncu summary, if present."""
+    path = os.path.join(ROOT, "profiles", "traffic.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        return d.get(f"{a.model}/{a.dtype}/K={a.K}")
+    except (OSError, ValueError):
+        return None
+
+
+def run_sweep(a, jb, table, mids, stream):
+    import torch
+    import synthetic
+    out = []
+    N = table.numel
+    for K in [int(k) for k in a.sweep.split(",") if k]:
+        seeds = jb.seeds_array([(int(m), 7, 0) for m in synthetic.machine_ids(K, 910)])
+        q = synthetic.byte_codes(K, 910)
+        reps = 3 if K <= 64 else 2
+        jb.jb_apply_updates(table, seeds, q, a.lr, 1.0, a.qscale, stream)
+        x0, x1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        x0.record(stream)
+        for _ in range(reps):
+            jb.jb_apply_updates(table, seeds, q, a.lr, 1.0, a.qscale, stream)
+        x1.record(stream)
+        torch.cuda.synchronize()
+        ms = x0.elapsed_time(x1) / reps
+        out.append({"K": K, "update_ms": ms, "param_seed_per_s": N * K / (ms / 1e3),
+                    "hbm_gbs": 2 * table.tensors[0].element_size() * N / (ms / 1e3) / 1e9})
+    p0, p1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    p0.record(stream)
+    for i in range(4):
+        jb.jb_perturb(table, (1, 2, 3), a.eps if i % 2 == 0 else -a.eps, stream)
+    p1.record(stream)
+    torch.cuda.synchronize()
+    pms = p0.elapsed_time(p1) / 4
+    out.append({"perturb_ms": pms, "param_seed_per_s": N / (pms / 1e3),
+                "hbm_gbs": 2 * table.tensors[0].element_size() * N / (pms / 1e3) / 1e9})
+    if a.sweep_out:
+        with open(a.sweep_out, "w") as f:
+            for ln in out:
+                f.write(json.dumps(ln) + "\n")
+    return out
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,185 @@
+/*
+ * jb.h -- C ABI of the GB300 (sm_103a) seeded-perturbation library "libjb".
+ *
+ * The library implements the data-parallel hot path of the decentralized
+ * shared-randomness SPSA of "Just One Byte (per gradient)" (arXiv 2306.10015):
+ * regenerate a seeded Gaussian perturbation z over every model parameter, in
+ * registers, and apply it in place.
+ *
+ *   jb_perturb        PerturbParameters(theta, eps, s): theta_i += eps z_i
+ *                     (Algorithm 1, subroutine); called with +eps, -2 eps,
+ *                     +eps around the two loss evaluations of one SPSA sample
+ *                     (Algorithm 1, inference loop).
+ *   jb_apply_updates  the step update: every machine's (seed, one-byte
+ *                     projected gradient) pair applied with weight
+ *                     -grad * eta / numel(all_grads) in machine-timestamp
+ *                     order (Section 2, "Applying collected scalar projected
+ *                     gradients"; Algorithm 1), fused into one read and one
+ *                     write of theta.
+ *   jb_quantize_grad  the one-byte projected gradient, "signed log of the
+ *   jb_dequantize_grad gradient clipped to +-127" (Section 3, Training Speed).
+ *
+ * ---------------------------------------------------------------------------
+ * Random stream. The paper names no generator (Appendix B notes that PyTorch's
+ * CUDA generator is not reproducible across GPU types). This library fixes:
+ *   - Philox4x32-10 (Salmon et al., SC 2011) with key = (lo, hi) words of
+ *     seed.machine_id and counter = (lo(b), hi(b), seed.step, seed.sample_id)
+ *     for block b = e >> 2 of global element index e; element e uses word
+ *     e & 3 of its block;
+ *   - Box-Muller on the word pairs (0,1) and (2,3) of a block:
+ *     u_a = ((x_a >> 9) + 1/2) 2^-23, u_b = ((x_b >> 8) + 1/2) 2^-24,
+ *     r = sqrt(-2 ln u_a); even element r cos(2 pi u_b), odd r sin(2 pi u_b).
+ *   z depends only on (seed, e): never on the tensor split, the launch
+ *   geometry or the GPU run, so every replica regenerates identical noise.
+ *
+ * Global element index. Each tensor ("segment") carries flat_offset, the
+ * global index of its element 0: element i of the segment is e = flat_offset
+ * + i. Every replica must use the same table (part of the shared model
+ * layout). Recommended: flat_offset of tensor t = align_up(flat_offset of
+ * t-1 + numel of t-1, 8) in named_parameters() order. The vectorised path
+ * needs (ptr - flat_offset * sizeof(T)) to be a multiple of 16 bytes; other
+ * segments are still handled, element by element, at lower speed.
+ *
+ * Arithmetic. z in fp32; |z| <= sqrt(48 ln 2) = 5.77. Perturb: one fp32 fused
+ * multiply-add theta + eps z, then one rounding to the storage type (nearest,
+ * ties to even). Update: acc = 0; for each pair k in canonical order
+ * acc = fma(c_k, z_k, acc) in fp32; theta <- round(theta + acc) once. No
+ * flush-to-zero. Results are bitwise repeatable.
+ *
+ * Memory and streams. The caller owns all device memory (e.g. torch
+ * tensors). The library copies the host arrays it is given (segments, seeds,
+ * codes) during the call, keeps no pointer to them, allocates no device
+ * memory and holds no state between calls other than a per-device cache of
+ * the SM count. Work is enqueued on `stream` (a cudaStream_t; NULL is the
+ * legacy default stream) and the call returns without waiting for it. Calls on
+ * different streams that touch the same parameters race.
+ *
+ * Errors. Every entry point returns a jb_status. Argument errors are detected
+ * before anything is enqueued, and then nothing is enqueued. JB_ERR_CUDA
+ * reports a launch failure seen by cudaGetLastError; faults during execution
+ * surface at the caller's next synchronisation. No exception, abort or exit
+ * crosses this interface.
+ */
+#ifndef JB_H
+#define JB_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+struct CUstream_st; /* cudaStream_t is struct CUstream_st* */
+
+typedef enum {
+    JB_OK = 0,
+    JB_ERR_INVALID_ARG = -1,      /* NULL pointer, negative count, bad scalar, overlap */
+    JB_ERR_UNSUPPORTED_DTYPE = -2,
+    JB_ERR_MISALIGNED = -3,       /* segment pointer not aligned to its element size */
+    JB_ERR_DUPLICATE_SEED = -4,   /* two pairs with the same (machine_id, step, sample_id) */
+    JB_ERR_CUDA = -5,             /* a CUDA runtime call or launch failed */
+    JB_ERR_RANGE = -6,            /* a coefficient -lr deq(q) / denom is not finite in fp32 */
+    JB_ERR_TOO_MANY_SEEDS = -7    /* K above jb_max_seeds_per_call() */
+} jb_status;
+
+typedef enum { JB_F32 = 0, JB_BF16 = 1 } jb_dtype;
+
+/* One parameter tensor: `numel` contiguous elements of the call's dtype at
+ * device address `ptr` (caller-owned), element i having global index
+ * flat_offset + i. Segments must not overlap in memory nor in global index. */
+typedef struct {
+    void* ptr;
+    uint64_t numel;
+    uint64_t flat_offset;
+} jb_segment;
+
+/* Seed s = (machine start-time identifier, iteration, sample index) of
+ * Algorithm 1 ("s <- (self_time, t, length(projected_grads))"). 16 bytes. */
+typedef struct {
+    uint64_t machine_id;
+    uint32_t step;
+    uint32_t sample_id;
+} jb_seed;
+
+/*
+ * jb_perturb -- PerturbParameters(theta, eps, s) (Algorithm 1, subroutine):
+ * for every element e of every segment, theta_e <- round_T(fma(eps, z_e(seed),
+ * theta_e)). In place, asynchronous on `stream`.
+ *   segs, n_segs  segment table (host array, copied); n_segs = 0 is a no-op.
+ *   dtype         JB_F32 or JB_BF16 for all segments.
+ *   eps           finite perturbation scale (use +eps, -2 eps, +eps for one
+ *                 SPSA sample; eps = 0 still rewrites theta unchanged).
+ */
+int jb_perturb(const jb_segment* segs, int n_segs, int dtype, jb_seed seed, float eps,
+               struct CUstream_st* stream);
+
+/*
+ * jb_apply_updates -- apply K machines' projected gradients in one pass
+ * (Section 2; Algorithm 1, gradient application):
+ *   theta_e <- round_T(theta_e + sum_k c_k z_e(seeds[k])),
+ *   c_k = (float)(-(double)lr * deq(q[k]) / (double)denom) with deq as in
+ *   jb_dequantize_grad, pairs taken in ascending (machine_id, step,
+ *   sample_id) order whatever order they are passed in.
+ * The paper divides by numel(all_grads) (denom = K); Section 4 scales the
+ * learning rate with sqrt(#perturbations): denom is therefore the caller's.
+ *   seeds, q, K   host arrays of K pairs (copied). K = 0 is a no-op.
+ *                 K <= jb_max_seeds_per_call(); duplicates are an error.
+ *   lr, denom     finite, denom != 0. qscale: S > 0 of the byte code.
+ * Returns JB_ERR_RANGE (nothing enqueued) if some c_k is not finite in fp32.
+ */
+int jb_apply_updates(const jb_segment* segs, int n_segs, int dtype, const jb_seed* seeds,
+                     const int8_t* q, int K, float lr, float denom, float qscale,
+                     struct CUstream_st* stream);
+
+/*
+ * jb_quantize_grad -- one-byte projected gradient (Section 3, Training
+ * Speed: signed log of the gradient, clipped to +-127). Host only, pure:
+ *   *out = sign(g) * min(127, round_half_away(qscale * ln(1 + |g|))),
+ *   NaN -> 0, +-inf -> +-127. qscale must be finite and > 0.
+ */
+int jb_quantize_grad(double g, float qscale, int8_t* out);
+
+/*
+ * jb_dequantize_grad -- inverse of the byte code, host only, pure:
+ *   *out = (float)(sign(q) * expm1(min(|q|, 127) / qscale)) (code -128 reads as
+ *   -127). Computed in double, rounded once; may be +-inf for small qscale.
+ */
+int jb_dequantize_grad(int8_t q, float qscale, float* out);
+
+/* Largest K accepted by jb_apply_updates in one call (the pairs travel in the
+ * kernel's parameter space). */
+int jb_max_seeds_per_call(void);
+
+/* Static description of a status code. Never NULL. */
+const char* jb_status_string(int status);
+
+/* ---------------------------------------------------------------------------
+ * Test hooks (not on the hot path). Device buffers are caller-owned.
+ * ------------------------------------------------------------------------- */
+
+/* d_out[4 i + w] = word w of Philox block first_block + i under `seed`. */
+int jb_debug_philox(jb_seed seed, uint64_t first_block, uint64_t n_blocks, uint32_t* d_out,
+                    struct CUstream_st* stream);
+
+/* d_out[i] = z of global element first_elem + i under `seed` (fp32). */
+int jb_debug_gaussian(jb_seed seed, uint64_t first_elem, uint64_t n, float* d_out,
+                      struct CUstream_st* stream);
+
+/* Box-Muller of raw word pairs: d_out[2 i], d_out[2 i + 1] = z of the even and
+ * odd element for words (d_words[2 i], d_words[2 i + 1]). */
+int jb_debug_box_muller(const uint32_t* d_words, uint64_t n_pairs, float* d_out,
+                        struct CUstream_st* stream);
+
+/* jb_perturb / jb_apply_updates with an explicit number of CTAs (0 = the
+ * default persistent grid); results must not depend on it. */
+int jb_perturb_with_grid(const jb_segment* segs, int n_segs, int dtype, jb_seed seed, float eps,
+                         int grid_ctas, struct CUstream_st* stream);
+int jb_apply_updates_with_grid(const jb_segment* segs, int n_segs, int dtype,
+                               const jb_seed* seeds, const int8_t* q, int K, float lr,
+                               float denom, float qscale, int grid_ctas,
+                               struct CUstream_st* stream);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* JB_H */

@@ -1,0 +1,253 @@
+// jb_capi.cpp -- the C ABI of libjb (declared in include/jb.h).
+//
+// Host side of the hot path: argument checks, the canonical (machine id,
+// step, sample id) order of the pairs (Section 2: gradients are applied in
+// machine-timestamp order), the per-pair coefficients c_k = -lr deq(q_k) /
+// denom (Algorithm 1: weight -grad * eta / numel(all_grads)), the one-byte
+// code (Section 3, Training Speed), and the packing of segments and pairs
+// into kernel launches. Every element-wise step runs in the CUDA kernels.
+#include <algorithm>
+#include <cmath>
+#include <cstring>
+#include <vector>
+
+#include "jb.h"
+#include "jb_internal.h"
+
+#define JB_EXPORT extern "C" __attribute__((visibility("default")))
+
+namespace {
+
+constexpr uint64_t kMaxIndex = 1ull << 62;  // global element indices stay below this
+
+struct Seg {
+    uint64_t ptr, fo, n;
+};
+
+size_t elem_size(int dtype) { return dtype == JB_F32 ? 4 : 2; }
+int elems_per_vec(int dtype) { return dtype == JB_F32 ? 4 : 8; }
+
+// Checks the segment table; drops empty segments. Overlap in memory or in
+// global index is an argument error.
+int collect_segments(const jb_segment* segs, int n_segs, int dtype, std::vector<Seg>& out) {
+    if (dtype != JB_F32 && dtype != JB_BF16) return JB_ERR_UNSUPPORTED_DTYPE;
+    if (n_segs < 0 || (n_segs > 0 && segs == nullptr)) return JB_ERR_INVALID_ARG;
+    const uint64_t es = elem_size(dtype);
+    out.clear();
+    out.reserve(static_cast<size_t>(n_segs));
+    for (int i = 0; i < n_segs; ++i) {
+        const jb_segment& s = segs[i];
+        if (s.numel == 0) continue;
+        const uint64_t p = reinterpret_cast<uint64_t>(s.ptr);
+        if (p == 0) return JB_ERR_INVALID_ARG;
+        if (p % es != 0) return JB_ERR_MISALIGNED;
+        if (s.numel > kMaxIndex || s.flat_offset > kMaxIndex - s.numel) return JB_ERR_INVALID_ARG;
+        if (p > UINT64_MAX - s.numel * es) return JB_ERR_INVALID_ARG;
+        out.push_back({p, s.flat_offset, s.numel});
+    }
+    std::vector<Seg> by_fo(out), by_ptr(out);
+    std::sort(by_fo.begin(), by_fo.end(), [](const Seg& a, const Seg& b) { return a.fo < b.fo; });
+    for (size_t i = 1; i < by_fo.size(); ++i)
+        if (by_fo[i - 1].fo + by_fo[i - 1].n > by_fo[i].fo) return JB_ERR_INVALID_ARG;
+    std::sort(by_ptr.begin(), by_ptr.end(), [](const Seg& a, const Seg& b) { return a.ptr < b.ptr; });
+    for (size_t i = 1; i < by_ptr.size(); ++i)
+        if (by_ptr[i - 1].ptr + by_ptr[i - 1].n * es > by_ptr[i].ptr) return JB_ERR_INVALID_ARG;
+    return JB_OK;
+}
+
+// Fills params.segs / n_segs / n_vec with segments [first, first + count).
+template <typename P>
+void pack_segments(const std::vector<Seg>& segs, size_t first, size_t count, int dtype, P& params) {
+    const uint64_t E = static_cast<uint64_t>(elems_per_vec(dtype));
+    const uint64_t es = elem_size(dtype);
+    uint64_t vec = 0;
+    for (size_t i = 0; i < count; ++i) {
+        const Seg& s = segs[first + i];
+        jb::SegParam& g = params.segs[i];
+        const uint64_t v_begin = s.fo / E;
+        const uint64_t v_end = (s.fo + s.n + E - 1) / E;
+        // 16-byte vectors of the segment line up with element groups whose global
+        // index is a multiple of E iff ptr - fo * sizeof(T) is 16-byte aligned.
+        const bool aligned = ((s.ptr - s.fo * es) & 15ull) == 0;
+        g.ptr = s.ptr | (aligned ? 1ull : 0ull);
+        g.fo = s.fo;
+        g.n = s.n;
+        g.vec0 = vec;
+        vec += v_end - v_begin;
+    }
+    params.n_segs = static_cast<uint32_t>(count);
+    params.n_vec = vec;
+}
+
+jb::SeedParam seed_param(const jb_seed& s, float coef) {
+    jb::SeedParam p;
+    p.k0 = static_cast<uint32_t>(s.machine_id);
+    p.k1 = static_cast<uint32_t>(s.machine_id >> 32);
+    p.step = s.step;
+    p.sample = s.sample_id;
+    p.coef = coef;
+    return p;
+}
+
+bool seed_less(const jb_seed& a, const jb_seed& b) {
+    if (a.machine_id != b.machine_id) return a.machine_id < b.machine_id;
+    if (a.step != b.step) return a.step < b.step;
+    return a.sample_id < b.sample_id;
+}
+
+bool seed_equal(const jb_seed& a, const jb_seed& b) {
+    return a.machine_id == b.machine_id && a.step == b.step && a.sample_id == b.sample_id;
+}
+
+double dequantize(int8_t q, double qscale) {
+    int m = q < 0 ? -static_cast<int>(q) : static_cast<int>(q);
+    if (m > 127) m = 127;
+    const double v = std::expm1(static_cast<double>(m) / qscale);
+    return q < 0 ? -v : v;
+}
+
+int cuda_status(cudaError_t e) { return e == cudaSuccess ? JB_OK : JB_ERR_CUDA; }
+
+int perturb_impl(const jb_segment* segs, int n_segs, int dtype, jb_seed seed, float eps,
+                 int grid_ctas, cudaStream_t stream) {
+    std::vector<Seg> v;
+    int rc = collect_segments(segs, n_segs, dtype, v);
+    if (rc != JB_OK) return rc;
+    if (!std::isfinite(eps)) return JB_ERR_INVALID_ARG;
+    if (v.empty()) return JB_OK;
+    static thread_local jb::PerturbParams params;  // ~32 KB: keep it off the stack
+    params.n_seeds = 1;
+    params.seeds[0] = seed_param(seed, eps);
+    for (size_t first = 0; first < v.size(); first += jb::kMaxSegsPerturb) {
+        const size_t count = std::min<size_t>(jb::kMaxSegsPerturb, v.size() - first);
+        pack_segments(v, first, count, dtype, params);
+        rc = cuda_status(jb::launch_perturb(params, dtype, grid_ctas, stream));
+        if (rc != JB_OK) return rc;
+    }
+    return JB_OK;
+}
+
+int update_impl(const jb_segment* segs, int n_segs, int dtype, const jb_seed* seeds,
+                const int8_t* q, int K, float lr, float denom, float qscale, int grid_ctas,
+                cudaStream_t stream) {
+    std::vector<Seg> v;
+    int rc = collect_segments(segs, n_segs, dtype, v);
+    if (rc != JB_OK) return rc;
+    if (K < 0 || (K > 0 && (seeds == nullptr || q == nullptr))) return JB_ERR_INVALID_ARG;
+    if (!std::isfinite(lr) || !std::isfinite(denom) || denom == 0.0f || !std::isfinite(qscale) ||
+        !(qscale > 0.0f))
+        return JB_ERR_INVALID_ARG;
+    if (K > jb::kMaxSeedsPerLaunch) return JB_ERR_TOO_MANY_SEEDS;
+    if (K == 0) return JB_OK;
+
+    // Canonical order: ascending (machine id, step, sample id).
+    std::vector<int> order(static_cast<size_t>(K));
+    for (int k = 0; k < K; ++k) order[k] = k;
+    std::stable_sort(order.begin(), order.end(),
+                     [&](int a, int b) { return seed_less(seeds[a], seeds[b]); });
+    for (int k = 1; k < K; ++k)
+        if (seed_equal(seeds[order[k - 1]], seeds[order[k]])) return JB_ERR_DUPLICATE_SEED;
+
+    static thread_local jb::UpdateParams params;
+    params.n_seeds = static_cast<uint32_t>(K);
+    for (int k = 0; k < K; ++k) {
+        const int i = order[k];
+        const double c = -static_cast<double>(lr) * dequantize(q[i], static_cast<double>(qscale)) /
+                         static_cast<double>(denom);
+        const float cf = static_cast<float>(c);
+        if (!std::isfinite(cf)) return JB_ERR_RANGE;
+        params.seeds[k] = seed_param(seeds[i], cf);
+    }
+    if (v.empty()) return JB_OK;
+    for (size_t first = 0; first < v.size(); first += jb::kMaxSegsUpdate) {
+        const size_t count = std::min<size_t>(jb::kMaxSegsUpdate, v.size() - first);
+        pack_segments(v, first, count, dtype, params);
+        rc = cuda_status(jb::launch_update(params, dtype, grid_ctas, stream));
+        if (rc != JB_OK) return rc;
+    }
+    return JB_OK;
+}
+
+}  // namespace
+
+JB_EXPORT int jb_perturb(const jb_segment* segs, int n_segs, int dtype, jb_seed seed, float eps,
+                         struct CUstream_st* stream) {
+    return perturb_impl(segs, n_segs, dtype, seed, eps, 0, stream);
+}
+
+JB_EXPORT int jb_perturb_with_grid(const jb_segment* segs, int n_segs, int dtype, jb_seed seed,
+                                   float eps, int grid_ctas, struct CUstream_st* stream) {
+    return perturb_impl(segs, n_segs, dtype, seed, eps, grid_ctas, stream);
+}
+
+JB_EXPORT int jb_apply_updates(const jb_segment* segs, int n_segs, int dtype, const jb_seed* seeds,
+                               const int8_t* q, int K, float lr, float denom, float qscale,
+                               struct CUstream_st* stream) {
+    return update_impl(segs, n_segs, dtype, seeds, q, K, lr, denom, qscale, 0, stream);
+}
+
+JB_EXPORT int jb_apply_updates_with_grid(const jb_segment* segs, int n_segs, int dtype,
+                                         const jb_seed* seeds, const int8_t* q, int K, float lr,
+                                         float denom, float qscale, int grid_ctas,
+                                         struct CUstream_st* stream) {
+    return update_impl(segs, n_segs, dtype, seeds, q, K, lr, denom, qscale, grid_ctas, stream);
+}
+
+JB_EXPORT int jb_quantize_grad(double g, float qscale, int8_t* out) {
+    if (out == nullptr || !std::isfinite(qscale) || !(qscale > 0.0f)) return JB_ERR_INVALID_ARG;
+    if (std::isnan(g)) {
+        *out = 0;
+        return JB_OK;
+    }
+    double mag = std::isinf(g) ? 127.0
+                               : std::round(static_cast<double>(qscale) * std::log1p(std::fabs(g)));
+    if (mag > 127.0) mag = 127.0;
+    const int m = static_cast<int>(mag);
+    *out = static_cast<int8_t>(g < 0 ? -m : m);
+    return JB_OK;
+}
+
+JB_EXPORT int jb_dequantize_grad(int8_t q, float qscale, float* out) {
+    if (out == nullptr || !std::isfinite(qscale) || !(qscale > 0.0f)) return JB_ERR_INVALID_ARG;
+    *out = static_cast<float>(dequantize(q, static_cast<double>(qscale)));
+    return JB_OK;
+}
+
+JB_EXPORT int jb_max_seeds_per_call(void) { return jb::kMaxSeedsPerLaunch; }
+
+JB_EXPORT const char* jb_status_string(int status) {
+    switch (status) {
+        case JB_OK: return "ok";
+        case JB_ERR_INVALID_ARG: return "invalid argument";
+        case JB_ERR_UNSUPPORTED_DTYPE: return "unsupported dtype (use JB_F32 or JB_BF16)";
+        case JB_ERR_MISALIGNED: return "segment pointer not aligned to its element size";
+        case JB_ERR_DUPLICATE_SEED: return "duplicate (machine_id, step, sample_id) seed";
+        case JB_ERR_CUDA: return "CUDA runtime or launch error";
+        case JB_ERR_RANGE: return "update coefficient not finite in fp32";
+        case JB_ERR_TOO_MANY_SEEDS: return "more seeds than one call accepts";
+        default: return "unknown status";
+    }
+}
+
+JB_EXPORT int jb_debug_philox(jb_seed seed, uint64_t first_block, uint64_t n_blocks, uint32_t* d_out,
+                              struct CUstream_st* stream) {
+    if (n_blocks > 0 && d_out == nullptr) return JB_ERR_INVALID_ARG;
+    if (n_blocks > (1ull << 38)) return JB_ERR_INVALID_ARG;
+    if (reinterpret_cast<uint64_t>(d_out) & 15ull) return JB_ERR_MISALIGNED;  // one 16-byte store per block
+    return cuda_status(jb::launch_debug_philox(seed_param(seed, 0.0f), first_block, n_blocks, d_out,
+                                               stream));
+}
+
+JB_EXPORT int jb_debug_gaussian(jb_seed seed, uint64_t first_elem, uint64_t n, float* d_out,
+                                struct CUstream_st* stream) {
+    if (n > 0 && d_out == nullptr) return JB_ERR_INVALID_ARG;
+    if (n > (1ull << 38) || first_elem > kMaxIndex - n) return JB_ERR_INVALID_ARG;
+    return cuda_status(jb::launch_debug_gaussian(seed_param(seed, 0.0f), first_elem, n, d_out, stream));
+}
+
+JB_EXPORT int jb_debug_box_muller(const uint32_t* d_words, uint64_t n_pairs, float* d_out,
+                                  struct CUstream_st* stream) {
+    if (n_pairs > 0 && (d_words == nullptr || d_out == nullptr)) return JB_ERR_INVALID_ARG;
+    if (n_pairs > (1ull << 38)) return JB_ERR_INVALID_ARG;
+    return cuda_status(jb::launch_debug_box_muller(d_words, n_pairs, d_out, stream));
+}

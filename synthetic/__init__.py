@@ -2,9 +2,9 @@
 
 This module holds no arithmetic of the method itself (no random-number stream
 of the method, no Gaussian transform, no perturbation, no update, no byte
-codec). It only builds workload shapes and draws input values with numpy's own
-generators, so that the CUDA path and the CPU oracle can be fed identical
-bytes.
+codec). It only builds workload shapes and draws input values with numpy's or
+torch's own seeded generators, so that the CUDA path and the CPU oracle can be
+fed identical bytes.
 
 Workloads stand in for the paper's fine-tuning runs (OPT models on SST-2,
 Section 3): the hot path depends only on the parameter count, the dtype, the
@@ -161,3 +161,42 @@ def membership_schedule(n_steps: int, pool: int = 1024, max_active: int = 512, *
     for _ in range(n_steps):
         m = int(g.integers(1, max_active + 1))
         yield np.sort(g.choice(ids, size=m, replace=False))
+
+
+def opt_parameters(model: str, dtype, device="cuda", seed: int = MASTER_SEED):
+    """OPT-shaped parameter tensors on `device`, one allocation per tensor.
+
+    Weights and embeddings ~ N(0, 0.02), LayerNorm gains 1, biases 0, drawn
+    with torch's own seeded generator on the device (input generation only).
+    Returns (specs, tensors, flat_offsets).
+    """
+    import torch
+    specs = opt_tensors(model)
+    gen = torch.Generator(device=device)
+    gen.manual_seed(seed)
+    tensors = []
+    for s in specs:
+        t = torch.empty(s.numel, dtype=dtype, device=device)
+        if s.init == "normal":
+            t.normal_(0.0, 0.02, generator=gen)
+        elif s.init == "ones":
+            t.fill_(1.0)
+        else:
+            t.zero_()
+        tensors.append(t)
+    return specs, tensors, flat_offsets([s.numel for s in specs])
+
+
+def sample_positions(numels: Sequence[int], n_samples: int, *stream: int) -> List[np.ndarray]:
+    """Per-tensor sorted sample positions: the first and last element of every
+    tensor plus n_samples positions drawn uniformly over all elements."""
+    g = rng(501, *stream)
+    total = int(sum(numels))
+    flat = np.sort(g.integers(0, total, size=n_samples, dtype=np.int64))
+    bounds = np.cumsum([0] + [int(n) for n in numels])
+    out = []
+    for i, n in enumerate(numels):
+        lo, hi = np.searchsorted(flat, [bounds[i], bounds[i + 1]])
+        p = np.concatenate([[0, int(n) - 1], flat[lo:hi] - bounds[i]])
+        out.append(np.unique(p).astype(np.int64))
+    return out
