@@ -15,7 +15,10 @@
 
 namespace jb {
 
-constexpr int kThreads = 256;          // threads per CTA
+#ifndef JB_THREADS
+#define JB_THREADS 256
+#endif
+constexpr int kThreads = JB_THREADS;   // threads per CTA
 constexpr int kMaxSeedsPerLaunch = 512;
 constexpr int kMaxSegsUpdate = 700;    // 16 + 512 * 20 + 700 * 32 bytes
 constexpr int kMaxSegsPerturb = 1000;  // 16 + 24 + 1000 * 32 bytes

@@ -33,17 +33,42 @@
 namespace jb {
 namespace {
 
+#ifndef JB_V_F32
+#define JB_V_F32 4
+#endif
+#ifndef JB_V_BF16
+#define JB_V_BF16 2
+#endif
+#ifndef JB_MIN_CTAS_UPDATE  // 0: no occupancy hint to ptxas
+#define JB_MIN_CTAS_UPDATE 0
+#endif
+#ifndef JB_MIN_CTAS_PERTURB
+#define JB_MIN_CTAS_PERTURB 0
+#endif
+
+#ifndef JB_PIPE_F32
+#define JB_PIPE_F32 0
+#endif
+#ifndef JB_PIPE_BF16
+#define JB_PIPE_BF16 1
+#endif
+
+// Per storage type: elements per 16-byte vector, vectors per thread per warp tile,
+// and whether the update loop computes seed k + 1's Philox words while seed k is
+// transformed (measured faster for bf16, slower for fp32 at these tile sizes).
 template <typename T>
 struct Traits;
 template <>
 struct Traits<float> {
-    static constexpr int E = 4;  // elements per 16-byte vector
-    static constexpr int V = 4;  // vectors per thread per warp tile
+    static constexpr int E = 4;
+    static constexpr int V = JB_V_F32;
+    static constexpr bool PIPE = JB_PIPE_F32;
 };
 template <>
 struct Traits<__nv_bfloat16> {
     static constexpr int E = 8;
-    static constexpr int V = 2;
+    static constexpr int V = JB_V_BF16;
+    static constexpr bool PIPE = JB_PIPE_BF16;
 };
 
 __device__ __forceinline__ void load_vec(const float* p, float (&x)[4]) {
@@ -81,8 +106,48 @@ __device__ __forceinline__ Key seed_key(const SeedParam& s) {
     return k;
 }
 
+
+// Philox words of the B blocks of each of V vectors (blk[j] is a multiple of B, so
+// adding b never carries into the high word).
+template <int V, int B>
+__device__ __forceinline__ void tile_words(const SeedConst& sc, const uint64_t (&blk)[V],
+                                           uint4 (&w)[V][B]) {
+#pragma unroll
+    for (int j = 0; j < V; ++j)
+#pragma unroll
+        for (int b = 0; b < B; ++b)
+            w[j][b] = philox_block(sc, static_cast<uint32_t>(blk[j]) + b,
+                                   static_cast<uint32_t>(blk[j] >> 32));
+}
+
+// acc += c z for the Gaussians of the words w; accumulators are packed per block as
+// (elements 4b, 4b + 2) and (4b + 1, 4b + 3).
+template <int V, int B>
+__device__ __forceinline__ void tile_accumulate(const uint4 (&w)[V][B], float c,
+                                                float2 (&acc)[V][B][2]) {
+#pragma unroll
+    for (int j = 0; j < V; ++j)
+#pragma unroll
+        for (int b = 0; b < B; ++b) {
+            const GaussPair g = box_muller2(w[j][b]);
+            acc[j][b][0] = fma2<kPackO>(splat(c), g.even, acc[j][b][0]);
+            acc[j][b][1] = fma2<kPackO>(splat(c), g.odd, acc[j][b][1]);
+        }
+}
+
+template <typename T, bool UPDATE>
+struct MinCtas {
+    static constexpr int value = UPDATE ? JB_MIN_CTAS_UPDATE : JB_MIN_CTAS_PERTURB;
+};
+
 template <typename T, bool UPDATE, typename P>
-__global__ void __launch_bounds__(kThreads) seeded_kernel(const __grid_constant__ P p) {
+__global__ void
+#if JB_MIN_CTAS_UPDATE || JB_MIN_CTAS_PERTURB
+__launch_bounds__(kThreads, (MinCtas<T, UPDATE>::value > 0 ? MinCtas<T, UPDATE>::value : 1))
+#else
+__launch_bounds__(kThreads)
+#endif
+    seeded_kernel(const __grid_constant__ P p) {
     constexpr int E = Traits<T>::E;
     constexpr int V = Traits<T>::V;
     constexpr int B = E / 4;  // Philox blocks per vector
@@ -124,46 +189,60 @@ __global__ void __launch_bounds__(kThreads) seeded_kernel(const __grid_constant_
         }
 
         if constexpr (UPDATE) {
-            float acc[V][E];
+            float2 acc[V][B][2];
 #pragma unroll
             for (int j = 0; j < V; ++j)
 #pragma unroll
-                for (int t = 0; t < E; ++t) acc[j][t] = 0.0f;
+                for (int b = 0; b < B; ++b) acc[j][b][0] = acc[j][b][1] = make_float2(0.0f, 0.0f);
             const uint32_t K = p.n_seeds;
-            for (uint32_t k = 0; k < K; ++k) {
-                const Key key = seed_key(p.seeds[k]);
-                const float c = p.seeds[k].coef;
+            if constexpr (Traits<T>::PIPE) {
+                // Philox words of seed k + 1 are computed while seed k is transformed
+                // and accumulated: the integer-multiply work and the fp32 work of the
+                // two halves are independent and interleave in one instruction stream.
+                uint4 w[V][B];
+                tile_words<V, B>(seed_const(seed_key(p.seeds[0])), blk, w);
+                for (uint32_t k = 0; k < K; ++k) {
+                    const uint32_t kn = k + 1 < K ? k + 1 : k;
+                    uint4 wn[V][B];
+                    tile_words<V, B>(seed_const(seed_key(p.seeds[kn])), blk, wn);
+                    tile_accumulate<V, B>(w, p.seeds[k].coef, acc);
 #pragma unroll
-                for (int j = 0; j < V; ++j)
+                    for (int j = 0; j < V; ++j)
 #pragma unroll
-                    for (int b = 0; b < B; ++b) {
-                        const uint64_t bb = blk[j] + b;
-                        const float4 z = block_gaussians(key, static_cast<uint32_t>(bb),
-                                                         static_cast<uint32_t>(bb >> 32));
-                        acc[j][4 * b + 0] = __fmaf_rn(c, z.x, acc[j][4 * b + 0]);
-                        acc[j][4 * b + 1] = __fmaf_rn(c, z.y, acc[j][4 * b + 1]);
-                        acc[j][4 * b + 2] = __fmaf_rn(c, z.z, acc[j][4 * b + 2]);
-                        acc[j][4 * b + 3] = __fmaf_rn(c, z.w, acc[j][4 * b + 3]);
-                    }
+                        for (int b = 0; b < B; ++b) w[j][b] = wn[j][b];
+                }
+            } else {
+                for (uint32_t k = 0; k < K; ++k) {
+                    uint4 w[V][B];
+                    tile_words<V, B>(seed_const(seed_key(p.seeds[k])), blk, w);
+                    tile_accumulate<V, B>(w, p.seeds[k].coef, acc);
+                }
             }
 #pragma unroll
             for (int j = 0; j < V; ++j)
 #pragma unroll
-                for (int t = 0; t < E; ++t) x[j][t] = __fadd_rn(x[j][t], acc[j][t]);
+                for (int b = 0; b < B; ++b) {
+                    x[j][4 * b + 0] = __fadd_rn(x[j][4 * b + 0], acc[j][b][0].x);
+                    x[j][4 * b + 2] = __fadd_rn(x[j][4 * b + 2], acc[j][b][0].y);
+                    x[j][4 * b + 1] = __fadd_rn(x[j][4 * b + 1], acc[j][b][1].x);
+                    x[j][4 * b + 3] = __fadd_rn(x[j][4 * b + 3], acc[j][b][1].y);
+                }
         } else {
-            const Key key = seed_key(p.seeds[0]);
-            const float eps = p.seeds[0].coef;
+            const SeedConst sc = seed_const(seed_key(p.seeds[0]));
+            const float2 eps = splat(p.seeds[0].coef);
+            uint4 w[V][B];
+            tile_words<V, B>(sc, blk, w);
 #pragma unroll
             for (int j = 0; j < V; ++j)
 #pragma unroll
                 for (int b = 0; b < B; ++b) {
-                    const uint64_t bb = blk[j] + b;
-                    const float4 z = block_gaussians(key, static_cast<uint32_t>(bb),
-                                                     static_cast<uint32_t>(bb >> 32));
-                    x[j][4 * b + 0] = __fmaf_rn(eps, z.x, x[j][4 * b + 0]);
-                    x[j][4 * b + 1] = __fmaf_rn(eps, z.y, x[j][4 * b + 1]);
-                    x[j][4 * b + 2] = __fmaf_rn(eps, z.z, x[j][4 * b + 2]);
-                    x[j][4 * b + 3] = __fmaf_rn(eps, z.w, x[j][4 * b + 3]);
+                    const GaussPair g = box_muller2(w[j][b]);
+                    const float2 ev = fma2<kPackO>(eps, g.even, make_float2(x[j][4 * b + 0], x[j][4 * b + 2]));
+                    const float2 od = fma2<kPackO>(eps, g.odd, make_float2(x[j][4 * b + 1], x[j][4 * b + 3]));
+                    x[j][4 * b + 0] = ev.x;
+                    x[j][4 * b + 2] = ev.y;
+                    x[j][4 * b + 1] = od.x;
+                    x[j][4 * b + 3] = od.y;
                 }
         }
 
@@ -192,7 +271,8 @@ __global__ void debug_philox_kernel(SeedParam sp, uint64_t first, uint64_t n, ui
     const uint64_t i = static_cast<uint64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
     if (i >= n) return;
     const uint64_t b = first + i;
-    const uint4 w = philox_block(seed_key(sp), static_cast<uint32_t>(b), static_cast<uint32_t>(b >> 32));
+    const uint4 w = philox_block(seed_const(seed_key(sp)), static_cast<uint32_t>(b),
+                                 static_cast<uint32_t>(b >> 32));
     reinterpret_cast<uint4*>(out)[i] = w;
 }
 
@@ -201,17 +281,25 @@ __global__ void debug_gaussian_kernel(SeedParam sp, uint64_t first, uint64_t n, 
     if (i >= n) return;
     const uint64_t e = first + i;
     const uint64_t b = e >> 2;
-    const float4 z = block_gaussians(seed_key(sp), static_cast<uint32_t>(b), static_cast<uint32_t>(b >> 32));
+    const float4 z = block_gaussians(seed_const(seed_key(sp)), static_cast<uint32_t>(b),
+                                     static_cast<uint32_t>(b >> 32));
     const unsigned w = static_cast<unsigned>(e & 3u);
     out[i] = w == 0 ? z.x : (w == 1 ? z.y : (w == 2 ? z.z : z.w));
 }
 
 __global__ void debug_box_muller_kernel(const uint32_t* words, uint64_t n, float* out) {
-    const uint64_t i = static_cast<uint64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+    // the transform runs on two word pairs at once, as in the kernels above
+    const uint64_t i = 2 * (static_cast<uint64_t>(blockIdx.x) * blockDim.x + threadIdx.x);
     if (i >= n) return;
-    const float2 z = box_muller(words[2 * i], words[2 * i + 1]);
-    out[2 * i] = z.x;
-    out[2 * i + 1] = z.y;
+    const uint64_t i1 = i + 1 < n ? i + 1 : i;
+    const GaussPair g = box_muller2(make_uint4(words[2 * i], words[2 * i + 1], words[2 * i1],
+                                               words[2 * i1 + 1]));
+    out[2 * i] = g.even.x;
+    out[2 * i + 1] = g.odd.x;
+    if (i + 1 < n) {
+        out[2 * i + 2] = g.even.y;
+        out[2 * i + 3] = g.odd.y;
+    }
 }
 
 // Persistent grid: SM count x resident CTAs per SM, cached per device and kernel.
@@ -287,7 +375,7 @@ cudaError_t launch_debug_gaussian(SeedParam seed, uint64_t first, uint64_t n, fl
 
 cudaError_t launch_debug_box_muller(const uint32_t* words, uint64_t n, float* out, cudaStream_t s) {
     if (n == 0) return cudaSuccess;
-    debug_box_muller_kernel<<<blocks_for(n), 256, 0, s>>>(words, n, out);
+    debug_box_muller_kernel<<<blocks_for((n + 1) / 2), 256, 0, s>>>(words, n, out);
     return cudaGetLastError();
 }
 

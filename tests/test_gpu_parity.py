@@ -113,7 +113,8 @@ def test_gaussian_parity_1e8(jb):
 
 
 def test_box_muller_extremes(jb):
-    """The largest radii (u_a -> 0) with every angle class, and every angle at r max."""
+    """Every radius word at two angles, every angle word at the largest radius, and the
+    largest radii (u_a -> 0) with the angles nearest the axes."""
     ma = np.arange(0, 1 << 12, dtype=np.uint32)
     angles = np.concatenate([np.arange(0, 64, dtype=np.uint32),
                              (np.arange(4, dtype=np.uint32) << 22)[:, None].ravel(),
@@ -121,8 +122,12 @@ def test_box_muller_extremes(jb):
     xa = np.repeat(ma << 9, angles.size)
     xb = np.tile(angles << 8, ma.size)
     all_b = np.arange(0, 1 << 24, dtype=np.uint32) << 8
-    xa = np.concatenate([xa, np.zeros(all_b.size, np.uint32), np.full(4096, 0xFFFFFFFF, np.uint32)])
-    xb = np.concatenate([xb, all_b, np.arange(4096, dtype=np.uint32) << 12])
+    all_a = np.arange(0, 1 << 23, dtype=np.uint32) << 9
+    xa = np.concatenate([xa, np.zeros(all_b.size, np.uint32), np.full(4096, 0xFFFFFFFF, np.uint32),
+                         all_a, all_a])
+    # every radius word at the angle nearest 0 (cos ~ 1) and nearest pi/4 (|cos| = |sin|)
+    xb = np.concatenate([xb, all_b, np.arange(4096, dtype=np.uint32) << 12,
+                         np.zeros(all_a.size, np.uint32), np.full(all_a.size, 0x1FFFFF << 8, np.uint32)])
     words = np.stack([xa, xb], 1).reshape(-1)
     n = xa.size
     d_words = torch.from_numpy(words.view(np.int32)).cuda()
@@ -132,7 +137,9 @@ def test_box_muller_extremes(jb):
     got = out.cpu().numpy().astype(np.float64).reshape(n, 2)
     want = oracle.box_muller_pairs(words.reshape(n, 2))
     err = np.abs(got - want)
-    print(f"max |dz| at extreme radii and all angles: {err.max():.3e}")
+    rel = err / np.maximum(np.abs(want), 1e-30)
+    print(f"max |dz| over all radius words and all angle words: {err.max():.3e}, "
+          f"max relative {rel.max():.3e}")
     assert err.max() <= Z_ABS_TOL
     # relative accuracy of the small members (the zeros of cos and sin are exact in angle)
     small = np.abs(want) < 1e-3

@@ -165,18 +165,25 @@ def test_dynamic_membership_30b(jb):
     start = vals.copy()
     lr, qs = float(F32(1e-4)), 16.0
     Ks = []
+    allowance = np.zeros(idx.size)
     for t, active in enumerate(synthetic.membership_schedule(20)):
         seeds = [(int(m), t, 0) for m in active]
         q = synthetic.byte_codes(len(seeds), 700 + t)
         Ks.append(len(seeds))
         jb.jb_apply_updates(table, seeds, q, lr, float(len(seeds)), qs)
+        # each step may add one bf16 step of its operands plus the fp32 allowance
+        scale = update_scale(vals, idx, seeds, q, lr, float(len(seeds)), qs)
+        allowance += np.ldexp(1.0, np.frexp(scale)[1] - 8) + 2e-6 * scale
         vals = oracle.update_at(vals, idx, seeds, q, lr, float(len(seeds)), qs)
     torch.cuda.synchronize()
     got = gather(table.tensors, pos)
     d = np.abs(bf16_ord(got) - bf16_ord(vals))
-    hist = np.bincount(d.astype(np.int64))
-    print(f"K_t = {Ks}; sampled {idx.size}; bf16 step histogram {hist.tolist()}")
-    assert d.max() <= 2 and hist[0] >= 0.99 * d.size
+    hist = np.bincount(np.minimum(d, 64).astype(np.int64))
+    err = np.abs(as_f64(got) - as_f64(vals))
+    print(f"K_t = {Ks}; sampled {idx.size}; bf16 step histogram {hist.tolist()}; "
+          f"worst error / allowance {float((err / allowance).max()):.3f}")
+    assert np.all(err <= allowance)
+    assert hist[0] >= 0.99 * d.size
     assert not np.array_equal(got, start)
     del table
     free_cuda()
