@@ -61,6 +61,8 @@ def parse():
                     help="target CPU time of the oracle sample")
     ap.add_argument("--sweep", default="", help="comma list of K: time update/perturb per K")
     ap.add_argument("--sweep-out", default="", help="file for the sweep's JSON lines")
+    ap.add_argument("--next-legs", action="store_true",
+                    help="with --sweep: also time the backup-fused update and the replay")
     return ap.parse_args()
 
 
@@ -406,10 +408,67 @@ def run_sweep(a, jb, table, mids, stream):
     pms = p0.elapsed_time(p1) / 4
     out.append({"perturb_ms": pms, "param_seed_per_s": N / (pms / 1e3),
                 "hbm_gbs": 2 * table.tensors[0].element_size() * N / (pms / 1e3) / 1e9})
+    if a.next_legs:
+        out.extend(next_legs(a, jb, table, stream))
     if a.sweep_out:
         with open(a.sweep_out, "w") as f:
             for ln in out:
                 f.write(json.dumps(ln) + "\n")
+    return out
+
+
+def next_legs(a, jb, table, stream):
+    """The update from the weight backup (restore fused) against copy + update, and
+    a replay of T steps against T separate updates, on the benchmark's set."""
+    import torch
+    import synthetic
+    out = []
+    ev = lambda: torch.cuda.Event(enable_timing=True)
+    K = a.K
+    seeds = jb.seeds_array([(int(m), 9, 0) for m in synthetic.machine_ids(K, 920)])
+    q = synthetic.byte_codes(K, 920)
+    backup = jb.ParamTable([torch.empty_like(t) for t in table.tensors], table.flat_offsets)
+    for b, t in zip(backup.tensors, table.tensors):
+        b.copy_(t)
+    for mode in ("copy+update", "fused", "fused+refresh"):
+        def once():
+            if mode == "copy+update":
+                for b, t in zip(backup.tensors, table.tensors):
+                    t.copy_(b)
+                jb.jb_apply_updates(table, seeds, q, a.lr, 1.0, a.qscale, stream)
+            else:
+                jb.jb_apply_updates_from(backup, table, seeds, q, a.lr, 1.0, a.qscale,
+                                         write_src=(mode == "fused+refresh"), stream=stream)
+        once()
+        x0, x1 = ev(), ev()
+        x0.record(stream)
+        for _ in range(2):
+            once()
+        x1.record(stream)
+        torch.cuda.synchronize()
+        out.append({"leg": "restore+update", "mode": mode, "K": K, "ms": x0.elapsed_time(x1) / 2})
+    del backup
+    for T, Kt in ((16, 4), (64, 1)):
+        steps = []
+        for t in range(T):
+            sd = jb.seeds_array([(int(m), 100 + t, 0) for m in synthetic.machine_ids(Kt, 930, t)])
+            steps.append((sd, synthetic.byte_codes(Kt, 930, t), a.lr, float(Kt)))
+        for mode in ("sequential", "replay"):
+            def once():
+                if mode == "replay":
+                    jb.jb_replay_updates(table, steps, a.qscale, stream)
+                else:
+                    for sd, qq, lr, den in steps:
+                        jb.jb_apply_updates(table, sd, qq, lr, den, a.qscale, stream)
+            once()
+            x0, x1 = ev(), ev()
+            x0.record(stream)
+            once()
+            x1.record(stream)
+            torch.cuda.synchronize()
+            out.append({"leg": "replay", "mode": mode, "steps": T, "K_per_step": Kt,
+                        "ms": x0.elapsed_time(x1),
+                        "param_seed_per_s": table.numel * T * Kt / (x0.elapsed_time(x1) / 1e3)})
     return out
 
 

@@ -132,6 +132,38 @@ int jb_apply_updates(const jb_segment* segs, int n_segs, int dtype, const jb_see
                      struct CUstream_st* stream);
 
 /*
+ * jb_apply_updates_from -- the step update applied to the weight backup, fused
+ * with the restore (Algorithm 1: theta <- copy(theta_backup), then every
+ * machine's gradients; Section 2: the backup avoids the drift of theta + z - z):
+ *   dst_e <- round_T(src_e + sum_k c_k z_e(seeds[k])), one read of src and one
+ *   write of dst per element (and one more write of src when write_src != 0, so
+ *   the next iteration's backup is refreshed in the same pass).
+ * Same pairs, coefficients, canonical order and rounding as jb_apply_updates;
+ * K = 0 copies src to dst.
+ *   src, dst   tables of n_segs segments: dst[i] has the numel and flat_offset of
+ *              src[i]; dst[i] is either src[i] itself or overlaps no source and
+ *              no other destination.
+ */
+int jb_apply_updates_from(const jb_segment* src, const jb_segment* dst, int n_segs, int dtype,
+                          const jb_seed* seeds, const int8_t* q, int K, float lr, float denom,
+                          float qscale, int write_src, struct CUstream_st* stream);
+
+/*
+ * jb_replay_updates -- a late joiner's catch-up (Appendix B): after downloading
+ * the weights, apply the projected gradients of every iteration it missed. Step
+ * t holds step_sizes[t] pairs (consecutive in seeds/q) and its own lr[t] and
+ * denom[t]; steps are applied in order, each rounded to the storage type as
+ * jb_apply_updates would round it, so the result is bitwise that of n_steps
+ * successive jb_apply_updates calls -- but theta is read and written once per
+ * launch instead of once per step. A step holds at most
+ * jb_max_seeds_per_call() pairs; steps are packed into launches of at most
+ * that many pairs.
+ */
+int jb_replay_updates(const jb_segment* segs, int n_segs, int dtype, const jb_seed* seeds,
+                      const int8_t* q, const int* step_sizes, int n_steps, const float* lr,
+                      const float* denom, float qscale, struct CUstream_st* stream);
+
+/*
  * jb_quantize_grad -- one-byte projected gradient (Section 3, Training
  * Speed: signed log of the gradient, clipped to +-127). Host only, pure:
  *   *out = sign(g) * min(127, round_half_away(qscale * ln(1 + |g|))),

@@ -6,6 +6,10 @@ streams. The functions keep the C names:
 
 * ``jb_perturb``        PerturbParameters(theta, eps, s) (Algorithm 1, subroutine)
 * ``jb_apply_updates``  the fused K-pair step update (Section 2; Algorithm 1)
+* ``jb_apply_updates_from``  the same update read from the weight backup, with the
+  restore of Algorithm 1 fused in
+* ``jb_replay_updates``  several steps' updates in one pass (a late joiner's
+  catch-up, Appendix B)
 * ``jb_quantize_grad`` / ``jb_dequantize_grad``  the one-byte projected
   gradient (Section 3, Training Speed)
 
@@ -67,6 +71,9 @@ def lib() -> ctypes.CDLL:
             L.jb_apply_updates.argtypes = [vp, i32, i32, vp, vp, i32, f32, f32, f32, vp]
             L.jb_apply_updates_with_grid.argtypes = [vp, i32, i32, vp, vp, i32, f32, f32, f32,
                                                      i32, vp]
+            L.jb_apply_updates_from.argtypes = [vp, vp, i32, i32, vp, vp, i32, f32, f32, f32,
+                                                i32, vp]
+            L.jb_replay_updates.argtypes = [vp, i32, i32, vp, vp, vp, i32, vp, vp, f32, vp]
             L.jb_quantize_grad.argtypes = [ctypes.c_double, f32, ctypes.POINTER(ctypes.c_int8)]
             L.jb_dequantize_grad.argtypes = [ctypes.c_int8, f32, ctypes.POINTER(ctypes.c_float)]
             L.jb_max_seeds_per_call.argtypes = []
@@ -76,7 +83,8 @@ def lib() -> ctypes.CDLL:
             L.jb_debug_gaussian.argtypes = [jb_seed, u64, u64, vp, vp]
             L.jb_debug_box_muller.argtypes = [vp, u64, vp, vp]
             for f in ("jb_perturb", "jb_perturb_with_grid", "jb_apply_updates",
-                      "jb_apply_updates_with_grid", "jb_quantize_grad", "jb_dequantize_grad",
+                      "jb_apply_updates_with_grid", "jb_apply_updates_from", "jb_replay_updates",
+                      "jb_quantize_grad", "jb_dequantize_grad",
                       "jb_max_seeds_per_call", "jb_debug_philox", "jb_debug_gaussian",
                       "jb_debug_box_muller"):
                 getattr(L, f).restype = i32
@@ -203,6 +211,40 @@ def jb_apply_updates(table: ParamTable, seeds, q, lr: float, denom: float, qscal
     _check(rc)
 
 
+def jb_apply_updates_from(src: ParamTable, dst: ParamTable, seeds, q, lr: float, denom: float,
+                          qscale: float, write_src: bool = False, stream=None) -> None:
+    """dst <- src - (lr / denom) sum_k deq(q_k) z(seed_k) in one pass (restore fused)."""
+    if src.n_segments != dst.n_segments or src.dtype != dst.dtype:
+        raise ValueError("source and destination tables differ")
+    s = seeds_array(seeds)
+    qa = np.ascontiguousarray(np.asarray(q, dtype=np.int8))
+    if qa.shape[0] != s.shape[0]:
+        raise ValueError("one byte code per seed")
+    K = s.shape[0]
+    _check(lib().jb_apply_updates_from(
+        src.segments, dst.segments, src.n_segments, src.dtype,
+        ctypes.c_void_p(s.ctypes.data if K else None), ctypes.c_void_p(qa.ctypes.data if K else None),
+        K, float(lr), float(denom), float(qscale), int(bool(write_src)), _stream(stream)))
+
+
+def jb_replay_updates(table: ParamTable, steps, qscale: float, stream=None) -> None:
+    """Apply several steps' updates in order, in place; steps = [(seeds, q, lr, denom), ...]."""
+    seeds = [seeds_array(st[0]) for st in steps]
+    codes = [np.asarray(st[1], dtype=np.int8) for st in steps]
+    sizes = np.array([len(x) for x in seeds], dtype=np.int32)
+    if any(len(c) != n for c, n in zip(codes, sizes)):
+        raise ValueError("one byte code per seed")
+    s = np.ascontiguousarray(np.concatenate(seeds) if len(seeds) else np.zeros(0, SEED_DTYPE))
+    qa = np.ascontiguousarray(np.concatenate(codes) if len(codes) else np.zeros(0, np.int8))
+    lr = np.array([float(st[2]) for st in steps], dtype=np.float32)
+    denom = np.array([float(st[3]) for st in steps], dtype=np.float32)
+    T = len(steps)
+    ptr = lambda a: ctypes.c_void_p(a.ctypes.data if a.size else None)
+    _check(lib().jb_replay_updates(table.segments, table.n_segments, table.dtype, ptr(s), ptr(qa),
+                                   ptr(sizes), T, ptr(lr), ptr(denom), float(qscale),
+                                   _stream(stream)))
+
+
 def jb_quantize_grad(g: float, qscale: float = 1.0) -> int:
     out = ctypes.c_int8()
     _check(lib().jb_quantize_grad(float(g), float(qscale), ctypes.byref(out)))
@@ -242,6 +284,7 @@ def jb_debug_box_muller(words, n_pairs: int, out, stream=None) -> None:
 __all__ = [
     "JB_OK", "JB_F32", "JB_BF16", "SEED_DTYPE", "JbError", "ParamTable", "jb_segment", "jb_seed",
     "lib", "seeds_array", "default_flat_offsets", "jb_perturb", "jb_apply_updates",
+    "jb_apply_updates_from", "jb_replay_updates",
     "jb_quantize_grad", "jb_dequantize_grad", "jb_max_seeds_per_call", "jb_status_string",
     "jb_debug_philox", "jb_debug_gaussian", "jb_debug_box_muller",
 ]

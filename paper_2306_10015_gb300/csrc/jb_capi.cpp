@@ -168,7 +168,170 @@ int update_impl(const jb_segment* segs, int n_segs, int dtype, const jb_seed* se
     return JB_OK;
 }
 
+// Destination table for src: same numel and flat offsets, element-aligned; each
+// destination either is its source or overlaps no source and no other destination.
+int collect_destinations(const jb_segment* src, const jb_segment* dst, int n_segs, int dtype,
+                         std::vector<uint64_t>& dptr) {
+    if (n_segs > 0 && dst == nullptr) return JB_ERR_INVALID_ARG;
+    const uint64_t es = elem_size(dtype);
+    struct Iv { uint64_t a, b; int owner; bool is_dst; };
+    std::vector<Iv> iv;
+    dptr.clear();
+    for (int i = 0; i < n_segs; ++i) {
+        if (src[i].numel == 0) {
+            if (dst[i].numel != 0) return JB_ERR_INVALID_ARG;
+            continue;
+        }
+        if (dst[i].numel != src[i].numel || dst[i].flat_offset != src[i].flat_offset)
+            return JB_ERR_INVALID_ARG;
+        const uint64_t p = reinterpret_cast<uint64_t>(dst[i].ptr);
+        if (p == 0) return JB_ERR_INVALID_ARG;
+        if (p % es != 0) return JB_ERR_MISALIGNED;
+        if (p > UINT64_MAX - dst[i].numel * es) return JB_ERR_INVALID_ARG;
+        dptr.push_back(p);
+        const uint64_t sp = reinterpret_cast<uint64_t>(src[i].ptr);
+        iv.push_back({sp, sp + src[i].numel * es, i, false});
+        if (p != sp) iv.push_back({p, p + src[i].numel * es, i, true});
+    }
+    std::sort(iv.begin(), iv.end(), [](const Iv& x, const Iv& y) { return x.a < y.a; });
+    for (size_t i = 1; i < iv.size(); ++i)
+        if (iv[i - 1].b > iv[i].a) return JB_ERR_INVALID_ARG;
+    return JB_OK;
+}
+
+// Shared by jb_apply_updates_from and jb_replay_updates: groups of pairs applied in
+// order, each group in canonical order with its own lr and denom, one rounding to
+// the storage type per group.
+int general_impl(const jb_segment* segs, const jb_segment* dsts, int n_segs, int dtype,
+                 const jb_seed* seeds, const int8_t* q, const int* group_sizes, int n_groups,
+                 const float* lr, const float* denom, float qscale, int write_src, int grid_ctas,
+                 cudaStream_t stream) {
+    std::vector<Seg> v;
+    int rc = collect_segments(segs, n_segs, dtype, v);
+    if (rc != JB_OK) return rc;
+    std::vector<uint64_t> dptr;
+    const bool out_of_place = dsts != nullptr;
+    if (out_of_place) {
+        rc = collect_destinations(segs, dsts, n_segs, dtype, dptr);
+        if (rc != JB_OK) return rc;
+    } else {
+        for (const Seg& g : v) dptr.push_back(g.ptr);
+    }
+    if (n_groups < 0 || (n_groups > 0 && (group_sizes == nullptr || lr == nullptr || denom == nullptr)))
+        return JB_ERR_INVALID_ARG;
+    if (!std::isfinite(qscale) || !(qscale > 0.0f)) return JB_ERR_INVALID_ARG;
+    long long total = 0;
+    for (int g = 0; g < n_groups; ++g) {
+        if (group_sizes[g] < 0) return JB_ERR_INVALID_ARG;
+        if (group_sizes[g] > jb::kMaxSeedsPerLaunch) return JB_ERR_TOO_MANY_SEEDS;
+        if (!std::isfinite(lr[g]) || !std::isfinite(denom[g]) || denom[g] == 0.0f)
+            return JB_ERR_INVALID_ARG;
+        total += group_sizes[g];
+    }
+    if (total > 0 && (seeds == nullptr || q == nullptr)) return JB_ERR_INVALID_ARG;
+
+    // every group in canonical order, with its coefficients
+    std::vector<jb::SeedParam> all(static_cast<size_t>(total));
+    std::vector<int> sizes;
+    long long base = 0;
+    for (int g = 0; g < n_groups; ++g) {
+        const int K = group_sizes[g];
+        std::vector<int> order(static_cast<size_t>(K));
+        for (int k = 0; k < K; ++k) order[k] = static_cast<int>(base) + k;
+        std::stable_sort(order.begin(), order.end(),
+                         [&](int a, int b) { return seed_less(seeds[a], seeds[b]); });
+        for (int k = 1; k < K; ++k)
+            if (seed_equal(seeds[order[k - 1]], seeds[order[k]])) return JB_ERR_DUPLICATE_SEED;
+        for (int k = 0; k < K; ++k) {
+            const int i = order[k];
+            const double c = -static_cast<double>(lr[g]) * dequantize(q[i], static_cast<double>(qscale)) /
+                             static_cast<double>(denom[g]);
+            const float cf = static_cast<float>(c);
+            if (!std::isfinite(cf)) return JB_ERR_RANGE;
+            all[static_cast<size_t>(base + k)] = seed_param(seeds[i], cf);
+        }
+        base += K;
+        if (K > 0) sizes.push_back(K);  // an empty group changes nothing
+    }
+    if (v.empty()) return JB_OK;
+    if (sizes.empty()) {
+        if (!out_of_place) return JB_OK;
+        sizes.clear();  // a pure copy: one launch with no group
+    }
+
+    static thread_local jb::GeneralParams params;
+    const uint64_t E = static_cast<uint64_t>(elems_per_vec(dtype));
+    const uint64_t es = elem_size(dtype);
+    // groups in launches of at most kMaxSeedsPerLaunch pairs / kMaxGroupsPerLaunch groups;
+    // after the first launch the destination holds the running value
+    size_t g0 = 0;
+    long long s0 = 0;
+    bool first = true;
+    do {
+        size_t g1 = g0;
+        long long n = 0;
+        while (g1 < sizes.size() && g1 - g0 < static_cast<size_t>(jb::kMaxGroupsPerLaunch) &&
+               n + sizes[g1] <= jb::kMaxSeedsPerLaunch)
+            n += sizes[g1++];
+        params.n_seeds = static_cast<uint32_t>(n);
+        params.n_groups = static_cast<uint32_t>(g1 - g0);
+        long long acc = 0;
+        for (size_t g = g0; g < g1; ++g) {
+            acc += sizes[g];
+            params.group_end[g - g0] = static_cast<uint16_t>(acc);
+        }
+        for (long long k = 0; k < n; ++k) params.seeds[k] = all[static_cast<size_t>(s0 + k)];
+        const bool last = g1 >= sizes.size();
+        // write_src comes with one group only (jb_apply_updates_from): one launch round
+        params.write_src = (write_src && last) ? 1u : 0u;
+        for (size_t first_seg = 0; first_seg < v.size(); first_seg += jb::kMaxSegsGeneral) {
+            const size_t count = std::min<size_t>(jb::kMaxSegsGeneral, v.size() - first_seg);
+            uint64_t vec = 0;
+            for (size_t i = 0; i < count; ++i) {
+                const Seg& sg = v[first_seg + i];
+                const uint64_t src_ptr = first ? sg.ptr : dptr[first_seg + i];
+                const uint64_t dst_ptr = dptr[first_seg + i];
+                jb::SegParamOut& g = params.segs[i];
+                const bool aligned = ((src_ptr - sg.fo * es) & 15ull) == 0 &&
+                                     ((dst_ptr - sg.fo * es) & 15ull) == 0;
+                g.ptr = src_ptr | (aligned ? 1ull : 0ull);
+                g.dst = dst_ptr;
+                g.fo = sg.fo;
+                g.n = sg.n;
+                g.vec0 = vec;
+                vec += (sg.fo + sg.n + E - 1) / E - sg.fo / E;
+            }
+            params.n_segs = static_cast<uint32_t>(count);
+            params.n_vec = vec;
+            rc = cuda_status(jb::launch_general(params, dtype, grid_ctas, stream));
+            if (rc != JB_OK) return rc;
+        }
+        s0 += n;
+        g0 = g1;
+        first = false;
+    } while (g0 < sizes.size());
+    return JB_OK;
+}
+
 }  // namespace
+
+JB_EXPORT int jb_apply_updates_from(const jb_segment* src, const jb_segment* dst, int n_segs,
+                                    int dtype, const jb_seed* seeds, const int8_t* q, int K,
+                                    float lr, float denom, float qscale, int write_src,
+                                    struct CUstream_st* stream) {
+    if (dst == nullptr && n_segs > 0) return JB_ERR_INVALID_ARG;
+    if (K < 0) return JB_ERR_INVALID_ARG;
+    return general_impl(src, dst, n_segs, dtype, seeds, q, &K, 1, &lr, &denom, qscale, write_src,
+                        0, stream);
+}
+
+JB_EXPORT int jb_replay_updates(const jb_segment* segs, int n_segs, int dtype, const jb_seed* seeds,
+                                const int8_t* q, const int* step_sizes, int n_steps,
+                                const float* lr, const float* denom, float qscale,
+                                struct CUstream_st* stream) {
+    return general_impl(segs, nullptr, n_segs, dtype, seeds, q, step_sizes, n_steps, lr, denom,
+                        qscale, 0, 0, stream);
+}
 
 JB_EXPORT int jb_perturb(const jb_segment* segs, int n_segs, int dtype, jb_seed seed, float eps,
                          struct CUstream_st* stream) {

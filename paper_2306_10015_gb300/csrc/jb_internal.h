@@ -51,11 +51,39 @@ using PerturbParams = LaunchParams<1, kMaxSegsPerturb>;
 static_assert(sizeof(UpdateParams) <= 32764, "update launch exceeds the parameter space");
 static_assert(sizeof(PerturbParams) <= 32764, "perturb launch exceeds the parameter space");
 
+// Generalised update: reads segment `ptr`, writes segment `dst` (and `ptr` too when
+// write_src), and applies the seeds in groups, rounding to the storage type after
+// each group: group g covers seeds [group_end[g - 1], group_end[g]).
+constexpr int kMaxGroupsPerLaunch = 512;
+constexpr int kMaxSegsGeneral = 512;
+
+struct SegParamOut {
+    uint64_t ptr;   // source; bit 0 set when source and destination take the vector path
+    uint64_t dst;   // destination
+    uint64_t fo;
+    uint64_t n;
+    uint64_t vec0;
+};
+
+struct GeneralParams {
+    uint32_t n_seeds;
+    uint32_t n_segs;
+    uint64_t n_vec;
+    uint32_t n_groups;
+    uint32_t write_src;
+    SeedParam seeds[kMaxSeedsPerLaunch];
+    uint16_t group_end[kMaxGroupsPerLaunch];
+    SegParamOut segs[kMaxSegsGeneral];
+};
+
+static_assert(sizeof(GeneralParams) <= 32764, "general launch exceeds the parameter space");
+
 enum DType { kF32 = 0, kBF16 = 1 };
 
 // Launchers (jb_kernels.cu). grid_ctas <= 0 selects the persistent grid.
 cudaError_t launch_update(const UpdateParams& p, int dtype, int grid_ctas, cudaStream_t s);
 cudaError_t launch_perturb(const PerturbParams& p, int dtype, int grid_ctas, cudaStream_t s);
+cudaError_t launch_general(const GeneralParams& p, int dtype, int grid_ctas, cudaStream_t s);
 cudaError_t launch_debug_philox(SeedParam seed, uint64_t first_block, uint64_t n_blocks,
                                 uint32_t* out, cudaStream_t s);
 cudaError_t launch_debug_gaussian(SeedParam seed, uint64_t first, uint64_t n, float* out,

@@ -46,6 +46,12 @@ namespace {
 #define JB_MIN_CTAS_PERTURB 0
 #endif
 
+#ifndef JB_VP_F32
+#define JB_VP_F32 4
+#endif
+#ifndef JB_VP_BF16
+#define JB_VP_BF16 2
+#endif
 #ifndef JB_PIPE_F32
 #define JB_PIPE_F32 0
 #endif
@@ -63,12 +69,14 @@ struct Traits<float> {
     static constexpr int E = 4;
     static constexpr int V = JB_V_F32;
     static constexpr bool PIPE = JB_PIPE_F32;
+    static constexpr int VP = JB_VP_F32;  // vectors per thread, perturb
 };
 template <>
 struct Traits<__nv_bfloat16> {
     static constexpr int E = 8;
     static constexpr int V = JB_V_BF16;
     static constexpr bool PIPE = JB_PIPE_BF16;
+    static constexpr int VP = JB_VP_BF16;
 };
 
 __device__ __forceinline__ void load_vec(const float* p, float (&x)[4]) {
@@ -140,6 +148,167 @@ struct MinCtas {
     static constexpr int value = UPDATE ? JB_MIN_CTAS_UPDATE : JB_MIN_CTAS_PERTURB;
 };
 
+// One thread's share of a warp tile: V vectors of E elements, as fp32 values,
+// with the segment, first Philox block and vector-path flag of each vector.
+template <typename T, int V>
+struct Tile {
+    static constexpr int E = Traits<T>::E;
+    float x[V][E];
+    uint32_t seg[V];
+    uint64_t blk[V];
+    bool full[V];
+};
+
+// Loads tile wt. The segment cursor s only moves forward: a thread's vector
+// indices grow from one call to the next.
+template <typename T, int V, typename P>
+__device__ __forceinline__ void load_tile(const P& p, uint64_t wt, uint32_t lane, uint32_t& s,
+                                          Tile<T, V>& tl) {
+    constexpr int E = Traits<T>::E;
+    const uint64_t n_vec = p.n_vec;
+    const uint32_t n_segs = p.n_segs;
+#pragma unroll
+    for (int j = 0; j < V; ++j) {
+        const uint64_t vi = wt * (32u * V) + 32u * j + lane;
+        const bool valid = vi < n_vec;
+        if (valid)
+            while (s + 1 < n_segs && p.segs[s + 1].vec0 <= vi) ++s;
+        tl.seg[j] = s;
+        const auto& g = p.segs[s];
+        const uint64_t e0 = (g.fo / E + (vi - g.vec0)) * E;
+        tl.blk[j] = e0 >> 2;
+        const int64_t i0 = static_cast<int64_t>(e0) - static_cast<int64_t>(g.fo);
+        const int64_t n = static_cast<int64_t>(g.n);
+        const T* base = reinterpret_cast<const T*>(g.ptr & ~1ull);
+        tl.full[j] = valid && (g.ptr & 1ull) && i0 >= 0 && i0 + E <= n;
+        if (tl.full[j]) {
+            load_vec(base + i0, tl.x[j]);
+        } else {
+#pragma unroll
+            for (int t = 0; t < E; ++t) {
+                const int64_t i = i0 + t;
+                tl.x[j][t] = (valid && i >= 0 && i < n) ? load_one(base + i) : 0.0f;
+            }
+        }
+    }
+}
+
+template <typename T, int V, bool TO_DST = false, typename P>
+__device__ __forceinline__ void store_tile(const P& p, uint64_t wt, uint32_t lane,
+                                           const Tile<T, V>& tl) {
+    constexpr int E = Traits<T>::E;
+#pragma unroll
+    for (int j = 0; j < V; ++j) {
+        const uint64_t vi = wt * (32u * V) + 32u * j + lane;
+        if (vi >= p.n_vec) continue;
+        const auto& g = p.segs[tl.seg[j]];
+        T* base;
+        if constexpr (TO_DST) base = reinterpret_cast<T*>(g.dst);
+        else base = reinterpret_cast<T*>(g.ptr & ~1ull);
+        const int64_t i0 = static_cast<int64_t>(tl.blk[j] << 2) - static_cast<int64_t>(g.fo);
+        if (tl.full[j]) {
+            store_vec(base + i0, tl.x[j]);
+        } else {
+            const int64_t n = static_cast<int64_t>(g.n);
+#pragma unroll
+            for (int t = 0; t < E; ++t) {
+                const int64_t i = i0 + t;
+                if (i >= 0 && i < n) store_one(base + i, tl.x[j][t]);
+            }
+        }
+    }
+}
+
+// acc = sum_{k in [kb, ke)} c_k z_k for the tile, in fp32, in seed order (ke > kb).
+template <typename T, int V, typename P>
+__device__ __forceinline__ void accumulate_range(const P& p, const uint64_t (&blk)[V], uint32_t kb,
+                                                 uint32_t ke, float2 (&acc)[V][Traits<T>::E / 4][2]) {
+    constexpr int B = Traits<T>::E / 4;  // Philox blocks per vector
+#pragma unroll
+    for (int j = 0; j < V; ++j)
+#pragma unroll
+        for (int b = 0; b < B; ++b) acc[j][b][0] = acc[j][b][1] = make_float2(0.0f, 0.0f);
+    if constexpr (Traits<T>::PIPE) {
+        // Philox words of seed k + 1 are computed while seed k is transformed and
+        // accumulated: the integer-multiply work and the fp32 work are independent
+        // and interleave in one instruction stream. The last seed is peeled.
+        uint4 w[V][B];
+        tile_words<V, B>(seed_const(seed_key(p.seeds[kb])), blk, w);
+        for (uint32_t k = kb; k + 1 < ke; ++k) {
+            uint4 wn[V][B];
+            tile_words<V, B>(seed_const(seed_key(p.seeds[k + 1])), blk, wn);
+            tile_accumulate<V, B>(w, p.seeds[k].coef, acc);
+#pragma unroll
+            for (int j = 0; j < V; ++j)
+#pragma unroll
+                for (int b = 0; b < B; ++b) w[j][b] = wn[j][b];
+        }
+        tile_accumulate<V, B>(w, p.seeds[ke - 1].coef, acc);
+    } else {
+        for (uint32_t k = kb; k < ke; ++k) {
+            uint4 w[V][B];
+            tile_words<V, B>(seed_const(seed_key(p.seeds[k])), blk, w);
+            tile_accumulate<V, B>(w, p.seeds[k].coef, acc);
+        }
+    }
+}
+
+// x += acc with one fp32 rounding; ROUND_T also rounds the sum to the storage type
+// (between the steps of a replay, where the next step reads the stored value).
+template <typename T, int V, bool ROUND_T>
+__device__ __forceinline__ void add_acc(Tile<T, V>& tl, const float2 (&acc)[V][Traits<T>::E / 4][2]) {
+    constexpr int B = Traits<T>::E / 4;
+#pragma unroll
+    for (int j = 0; j < V; ++j)
+#pragma unroll
+        for (int b = 0; b < B; ++b) {
+            float v0 = __fadd_rn(tl.x[j][4 * b + 0], acc[j][b][0].x);
+            float v2 = __fadd_rn(tl.x[j][4 * b + 2], acc[j][b][0].y);
+            float v1 = __fadd_rn(tl.x[j][4 * b + 1], acc[j][b][1].x);
+            float v3 = __fadd_rn(tl.x[j][4 * b + 3], acc[j][b][1].y);
+            if constexpr (ROUND_T && sizeof(T) == 2) {
+                v0 = __bfloat162float(__float2bfloat16_rn(v0));
+                v1 = __bfloat162float(__float2bfloat16_rn(v1));
+                v2 = __bfloat162float(__float2bfloat16_rn(v2));
+                v3 = __bfloat162float(__float2bfloat16_rn(v3));
+            }
+            tl.x[j][4 * b + 0] = v0;
+            tl.x[j][4 * b + 1] = v1;
+            tl.x[j][4 * b + 2] = v2;
+            tl.x[j][4 * b + 3] = v3;
+        }
+}
+
+// theta += sum_k c_k z_k over the tile, accumulated in fp32 in seed order.
+template <typename T, int V, typename P>
+__device__ __forceinline__ void update_tile(const P& p, Tile<T, V>& tl) {
+    float2 acc[V][Traits<T>::E / 4][2];
+    accumulate_range<T, V>(p, tl.blk, 0, p.n_seeds, acc);
+    add_acc<T, V, false>(tl, acc);
+}
+
+// theta <- fma(eps, z, theta) over the tile.
+template <typename T, int V, typename P>
+__device__ __forceinline__ void perturb_tile(const P& p, Tile<T, V>& tl) {
+    constexpr int B = Traits<T>::E / 4;
+    const SeedConst sc = seed_const(seed_key(p.seeds[0]));
+    const float2 eps = splat(p.seeds[0].coef);
+    uint4 w[V][B];
+    tile_words<V, B>(sc, tl.blk, w);
+#pragma unroll
+    for (int j = 0; j < V; ++j)
+#pragma unroll
+        for (int b = 0; b < B; ++b) {
+            const GaussPair g = box_muller2(w[j][b]);
+            const float2 ev = fma2<kPackO>(eps, g.even, make_float2(tl.x[j][4 * b + 0], tl.x[j][4 * b + 2]));
+            const float2 od = fma2<kPackO>(eps, g.odd, make_float2(tl.x[j][4 * b + 1], tl.x[j][4 * b + 3]));
+            tl.x[j][4 * b + 0] = ev.x;
+            tl.x[j][4 * b + 2] = ev.y;
+            tl.x[j][4 * b + 1] = od.x;
+            tl.x[j][4 * b + 3] = od.y;
+        }
+}
+
 template <typename T, bool UPDATE, typename P>
 __global__ void
 #if JB_MIN_CTAS_UPDATE || JB_MIN_CTAS_PERTURB
@@ -148,122 +317,45 @@ __launch_bounds__(kThreads, (MinCtas<T, UPDATE>::value > 0 ? MinCtas<T, UPDATE>:
 __launch_bounds__(kThreads)
 #endif
     seeded_kernel(const __grid_constant__ P p) {
-    constexpr int E = Traits<T>::E;
-    constexpr int V = Traits<T>::V;
-    constexpr int B = E / 4;  // Philox blocks per vector
+    constexpr int V = UPDATE ? Traits<T>::V : Traits<T>::VP;
     const uint32_t lane = threadIdx.x & 31u;
     const uint64_t warp = (static_cast<uint64_t>(blockIdx.x) * kThreads + threadIdx.x) >> 5;
     const uint64_t n_warps = (static_cast<uint64_t>(gridDim.x) * kThreads) >> 5;
     const uint64_t n_vec = p.n_vec;
-    const uint32_t n_segs = p.n_segs;
-    uint32_t s = 0;  // segment cursor: vector indices only grow within a thread
+    uint32_t s = 0;  // segment cursor
 
     for (uint64_t wt = warp; wt * (32u * V) < n_vec; wt += n_warps) {
-        float x[V][E];
-        uint32_t seg[V];
-        uint64_t blk[V];
-        bool full[V];
-#pragma unroll
-        for (int j = 0; j < V; ++j) {
-            const uint64_t vi = wt * (32u * V) + 32u * j + lane;
-            const bool valid = vi < n_vec;
-            if (valid)
-                while (s + 1 < n_segs && p.segs[s + 1].vec0 <= vi) ++s;
-            seg[j] = s;
-            const SegParam& g = p.segs[s];
-            const uint64_t e0 = (g.fo / E + (vi - g.vec0)) * E;
-            blk[j] = e0 >> 2;
-            const int64_t i0 = static_cast<int64_t>(e0) - static_cast<int64_t>(g.fo);
-            const int64_t n = static_cast<int64_t>(g.n);
-            T* base = reinterpret_cast<T*>(g.ptr & ~1ull);
-            full[j] = valid && (g.ptr & 1ull) && i0 >= 0 && i0 + E <= n;
-            if (full[j]) {
-                load_vec(base + i0, x[j]);
-            } else {
-#pragma unroll
-                for (int t = 0; t < E; ++t) {
-                    const int64_t i = i0 + t;
-                    x[j][t] = (valid && i >= 0 && i < n) ? load_one(base + i) : 0.0f;
-                }
-            }
-        }
+        Tile<T, V> tl;
+        load_tile<T, V>(p, wt, lane, s, tl);
+        if constexpr (UPDATE) update_tile<T, V>(p, tl);
+        else perturb_tile<T, V>(p, tl);
+        store_tile<T, V>(p, wt, lane, tl);
+    }
+}
 
-        if constexpr (UPDATE) {
-            float2 acc[V][B][2];
-#pragma unroll
-            for (int j = 0; j < V; ++j)
-#pragma unroll
-                for (int b = 0; b < B; ++b) acc[j][b][0] = acc[j][b][1] = make_float2(0.0f, 0.0f);
-            const uint32_t K = p.n_seeds;
-            if constexpr (Traits<T>::PIPE) {
-                // Philox words of seed k + 1 are computed while seed k is transformed
-                // and accumulated: the integer-multiply work and the fp32 work of the
-                // two halves are independent and interleave in one instruction stream.
-                uint4 w[V][B];
-                tile_words<V, B>(seed_const(seed_key(p.seeds[0])), blk, w);
-                for (uint32_t k = 0; k < K; ++k) {
-                    const uint32_t kn = k + 1 < K ? k + 1 : k;
-                    uint4 wn[V][B];
-                    tile_words<V, B>(seed_const(seed_key(p.seeds[kn])), blk, wn);
-                    tile_accumulate<V, B>(w, p.seeds[k].coef, acc);
-#pragma unroll
-                    for (int j = 0; j < V; ++j)
-#pragma unroll
-                        for (int b = 0; b < B; ++b) w[j][b] = wn[j][b];
-                }
-            } else {
-                for (uint32_t k = 0; k < K; ++k) {
-                    uint4 w[V][B];
-                    tile_words<V, B>(seed_const(seed_key(p.seeds[k])), blk, w);
-                    tile_accumulate<V, B>(w, p.seeds[k].coef, acc);
-                }
-            }
-#pragma unroll
-            for (int j = 0; j < V; ++j)
-#pragma unroll
-                for (int b = 0; b < B; ++b) {
-                    x[j][4 * b + 0] = __fadd_rn(x[j][4 * b + 0], acc[j][b][0].x);
-                    x[j][4 * b + 2] = __fadd_rn(x[j][4 * b + 2], acc[j][b][0].y);
-                    x[j][4 * b + 1] = __fadd_rn(x[j][4 * b + 1], acc[j][b][1].x);
-                    x[j][4 * b + 3] = __fadd_rn(x[j][4 * b + 3], acc[j][b][1].y);
-                }
-        } else {
-            const SeedConst sc = seed_const(seed_key(p.seeds[0]));
-            const float2 eps = splat(p.seeds[0].coef);
-            uint4 w[V][B];
-            tile_words<V, B>(sc, blk, w);
-#pragma unroll
-            for (int j = 0; j < V; ++j)
-#pragma unroll
-                for (int b = 0; b < B; ++b) {
-                    const GaussPair g = box_muller2(w[j][b]);
-                    const float2 ev = fma2<kPackO>(eps, g.even, make_float2(x[j][4 * b + 0], x[j][4 * b + 2]));
-                    const float2 od = fma2<kPackO>(eps, g.odd, make_float2(x[j][4 * b + 1], x[j][4 * b + 3]));
-                    x[j][4 * b + 0] = ev.x;
-                    x[j][4 * b + 2] = ev.y;
-                    x[j][4 * b + 1] = od.x;
-                    x[j][4 * b + 3] = od.y;
-                }
+// The generalised update: source -> destination (optionally also back to the
+// source), seeds applied in groups with a rounding to the storage type after each
+// group, exactly as successive in-place updates would round.
+template <typename T>
+__global__ void __launch_bounds__(kThreads) general_update_kernel(const __grid_constant__ GeneralParams p) {
+    constexpr int V = Traits<T>::V;
+    const uint32_t lane = threadIdx.x & 31u;
+    const uint64_t warp = (static_cast<uint64_t>(blockIdx.x) * kThreads + threadIdx.x) >> 5;
+    const uint64_t n_warps = (static_cast<uint64_t>(gridDim.x) * kThreads) >> 5;
+    uint32_t s = 0;
+    for (uint64_t wt = warp; wt * (32u * V) < p.n_vec; wt += n_warps) {
+        Tile<T, V> tl;
+        load_tile<T, V>(p, wt, lane, s, tl);
+        uint32_t kb = 0;
+        for (uint32_t g = 0; g < p.n_groups; ++g) {
+            const uint32_t ke = p.group_end[g];  // > kb: the host drops empty groups
+            float2 acc[V][Traits<T>::E / 4][2];
+            accumulate_range<T, V>(p, tl.blk, kb, ke, acc);
+            add_acc<T, V, true>(tl, acc);
+            kb = ke;
         }
-
-#pragma unroll
-        for (int j = 0; j < V; ++j) {
-            const uint64_t vi = wt * (32u * V) + 32u * j + lane;
-            if (vi >= n_vec) continue;
-            const SegParam& g = p.segs[seg[j]];
-            T* base = reinterpret_cast<T*>(g.ptr & ~1ull);
-            const int64_t i0 = static_cast<int64_t>(blk[j] << 2) - static_cast<int64_t>(g.fo);
-            if (full[j]) {
-                store_vec(base + i0, x[j]);
-            } else {
-                const int64_t n = static_cast<int64_t>(g.n);
-#pragma unroll
-                for (int t = 0; t < E; ++t) {
-                    const int64_t i = i0 + t;
-                    if (i >= 0 && i < n) store_one(base + i, x[j][t]);
-                }
-            }
-        }
+        store_tile<T, V, true>(p, wt, lane, tl);
+        if (p.write_src) store_tile<T, V, false>(p, wt, lane, tl);
     }
 }
 
@@ -304,7 +396,7 @@ __global__ void debug_box_muller_kernel(const uint32_t* words, uint64_t n, float
 
 // Persistent grid: SM count x resident CTAs per SM, cached per device and kernel.
 constexpr int kMaxDevices = 64;
-constexpr int kKernels = 4;
+constexpr int kKernels = 6;
 std::atomic<int> g_grid_cache[kMaxDevices][kKernels];
 
 template <typename K>
@@ -337,7 +429,8 @@ cudaError_t launch_seeded(const P& p, int slot, int grid_ctas, cudaStream_t stre
     if (grid <= 0) {
         cudaError_t err = persistent_grid(kernel, slot, &grid);
         if (err != cudaSuccess) return err;
-        constexpr uint64_t vec_per_cta = 32ull * Traits<T>::V * (kThreads / 32);
+        constexpr uint64_t vec_per_cta =
+            32ull * (UPDATE ? Traits<T>::V : Traits<T>::VP) * (kThreads / 32);
         const uint64_t needed = (p.n_vec + vec_per_cta - 1) / vec_per_cta;
         if (needed < static_cast<uint64_t>(grid)) grid = static_cast<int>(needed);
     }
@@ -350,6 +443,27 @@ cudaError_t launch_seeded(const P& p, int slot, int grid_ctas, cudaStream_t stre
 cudaError_t launch_update(const UpdateParams& p, int dtype, int grid_ctas, cudaStream_t s) {
     if (dtype == kF32) return launch_seeded<float, true>(p, 0, grid_ctas, s);
     return launch_seeded<__nv_bfloat16, true>(p, 1, grid_ctas, s);
+}
+
+template <typename T>
+cudaError_t launch_general_t(const GeneralParams& p, int slot, int grid_ctas, cudaStream_t stream) {
+    if (p.n_vec == 0) return cudaSuccess;
+    auto kernel = general_update_kernel<T>;
+    int grid = grid_ctas;
+    if (grid <= 0) {
+        cudaError_t err = persistent_grid(kernel, slot, &grid);
+        if (err != cudaSuccess) return err;
+        constexpr uint64_t vec_per_cta = 32ull * Traits<T>::V * (kThreads / 32);
+        const uint64_t needed = (p.n_vec + vec_per_cta - 1) / vec_per_cta;
+        if (needed < static_cast<uint64_t>(grid)) grid = static_cast<int>(needed);
+    }
+    kernel<<<grid, kThreads, 0, stream>>>(p);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_general(const GeneralParams& p, int dtype, int grid_ctas, cudaStream_t s) {
+    if (dtype == kF32) return launch_general_t<float>(p, 4, grid_ctas, s);
+    return launch_general_t<__nv_bfloat16>(p, 5, grid_ctas, s);
 }
 
 cudaError_t launch_perturb(const PerturbParams& p, int dtype, int grid_ctas, cudaStream_t s) {

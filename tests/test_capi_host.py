@@ -161,3 +161,35 @@ def test_opt_shapes_match_known_parameter_counts():
         L = synthetic.OPT_SHAPES[name][0]
         assert sum(x.numel for x in t) == n
         assert len(t) == 16 * L + 4
+
+
+def test_apply_from_and_replay_validation(jb):
+    import ctypes as C
+    E = {"inv": -1, "dup": -4, "many": -7}
+    src = _segs(jb, [(FAKE, 100, 0), (FAKE + 4096, 50, 104)])
+    s = jb.seeds_array([(1, 0, 0), (2, 0, 0)])
+    q = np.array([3, 4], dtype=np.int8)
+    sp, qp = C.c_void_p(s.ctypes.data), C.c_void_p(q.ctypes.data)
+    L = jb.lib()
+    call = lambda dst, K=2: L.jb_apply_updates_from(src, dst, 2, 0, sp, qp, K, 1e-3, 1.0, 16.0, 0, None)
+    assert call(None) == E["inv"]
+    assert call(_segs(jb, [(FAKE + 8192, 100, 0), (FAKE + 16384, 49, 104)])) == E["inv"]  # numel
+    assert call(_segs(jb, [(FAKE + 8192, 100, 1), (FAKE + 16384, 50, 104)])) == E["inv"]  # offset
+    assert call(_segs(jb, [(FAKE + 200, 100, 0), (FAKE + 16384, 50, 104)])) == E["inv"]   # overlaps src
+    assert call(_segs(jb, [(FAKE + 8192, 100, 0), (FAKE + 8200, 50, 104)])) == E["inv"]   # dsts overlap
+    assert call(_segs(jb, [(FAKE + 8192, 100, 0), (FAKE + 16384, 50, 104)]), K=-1) == E["inv"]
+    dup = jb.seeds_array([(1, 0, 0), (1, 0, 0)])
+    assert L.jb_apply_updates_from(src, src, 2, 0, C.c_void_p(dup.ctypes.data), qp, 2, 1e-3, 1.0,
+                                   16.0, 0, None) == E["dup"]
+    sizes = np.array([1, 1], dtype=np.int32)
+    lr = np.array([1e-3, 1e-3], dtype=np.float32)
+    den = np.array([1.0, 0.0], dtype=np.float32)
+    replay = lambda sz, d: L.jb_replay_updates(src, 2, 0, sp, qp, C.c_void_p(sz.ctypes.data), len(sz),
+                                               C.c_void_p(lr.ctypes.data), C.c_void_p(d.ctypes.data),
+                                               16.0, None)
+    assert replay(sizes, den) == E["inv"]                                  # denom 0 in step 1
+    assert replay(np.array([1, -1], np.int32), np.ones(2, np.float32)) == E["inv"]
+    big = np.array([600, 0], np.int32)
+    assert replay(big, np.ones(2, np.float32)) == E["many"]                # one step > 512 pairs
+    # two equal seeds in different steps are legal (only a step must be duplicate-free):
+    # validation passes and the call reaches the launch, which has no device here
