@@ -93,6 +93,10 @@ def lib() -> ctypes.CDLL:
             L.jbo_update_delta_at.argtypes = [vp, u64, vp, vp, ctypes.c_int, ctypes.c_double,
                                               ctypes.c_double, ctypes.c_double, vp]
             L.jbo_update_delta_at.restype = ctypes.c_int
+            L.jbo_window_hash.argtypes = [u64, u32p]
+            L.jbo_window_hash.restype = ctypes.c_uint64
+            L.jbo_checksum_segment.argtypes = [vp, ctypes.c_int, u64, u64]
+            L.jbo_checksum_segment.restype = ctypes.c_uint64
             L.jbo_set_threads.argtypes = [ctypes.c_int]
             L.jbo_get_threads.restype = ctypes.c_int
             _lib = L
@@ -267,6 +271,22 @@ def update_delta_at(idx: np.ndarray, seeds, q, lr: float, denom: float,
     _check(lib().jbo_update_delta_at(_ptr(i), i.size, _ptr(s), _ptr(qa), len(s), lr, denom,
                                      qscale, _ptr(out)))
     return out
+
+
+# --- model checksum ----------------------------------------------------------
+
+def window_hash(window: int, words) -> int:
+    w = (ctypes.c_uint32 * 4)(*[int(x) & 0xFFFFFFFF for x in words])
+    return int(lib().jbo_window_hash(int(window), w))
+
+
+def checksum(tensors, flat_offsets) -> int:
+    """Sum mod 2^64 of the per-segment window contributions (see jb_oracle.c)."""
+    total = 0
+    for t, fo in zip(tensors, flat_offsets):
+        a = np.ascontiguousarray(t)
+        total += int(lib().jbo_checksum_segment(_ptr(a), _dtype_code(a), a.size, int(fo)))
+    return total % (1 << 64)
 
 
 def set_threads(n: int) -> None:

@@ -322,6 +322,66 @@ int jbo_update_delta_at(const uint64_t* idx, uint64_t n, const jbo_seed* seeds, 
 }
 
 /* ------------------------------------------------------------------------ */
+/* Model checksum for ChecksumMatch (Algorithm 1: "check if hashed theta      */
+/* matches peer's"). The paper fixes no hash. Reading: the global element     */
+/* index space is cut into windows of 16 bytes of storage (8 bf16 or 4 fp32   */
+/* elements; window v = elements [vE, vE + E)). Each window that overlaps a   */
+/* segment contributes, per segment, the first four Philox4x32 rounds of its  */
+/* four storage words (elements outside the segment read as 0) under the key */
+/* (lo v, hi v) xor (0x6A09E667, 0xF3BCC908); the checksum is the sum mod     */
+/* 2^64 of (x1:x0) + (x3:x2) over all contributions. Four rounds carry every */
+/* input bit into every output word; the sum does not depend on the order in  */
+/* which windows are evaluated.                                               */
+/* ------------------------------------------------------------------------ */
+static void philox_rounds(uint32_t w[4], uint32_t k0, uint32_t k1, int rounds) {
+    for (int r = 0; r < rounds; ++r) {
+        if (r > 0) {
+            k0 += PHILOX_W0;
+            k1 += PHILOX_W1;
+        }
+        uint64_t p0 = (uint64_t)PHILOX_M0 * (uint64_t)w[0];
+        uint64_t p1 = (uint64_t)PHILOX_M1 * (uint64_t)w[2];
+        uint32_t y0 = (uint32_t)(p1 >> 32) ^ w[1] ^ k0;
+        uint32_t y2 = (uint32_t)(p0 >> 32) ^ w[3] ^ k1;
+        w[1] = (uint32_t)p1;
+        w[3] = (uint32_t)p0;
+        w[0] = y0;
+        w[2] = y2;
+    }
+}
+
+uint64_t jbo_window_hash(uint64_t window, const uint32_t words[4]) {
+    uint32_t w[4] = {words[0], words[1], words[2], words[3]};
+    philox_rounds(w, (uint32_t)window ^ 0x6A09E667u, (uint32_t)(window >> 32) ^ 0xF3BCC908u, 4);
+    return ((uint64_t)w[1] << 32 | w[0]) + ((uint64_t)w[3] << 32 | w[2]);
+}
+
+/* Contribution of one segment (values at global indices fo .. fo + n - 1). */
+uint64_t jbo_checksum_segment(const void* theta, int dtype, uint64_t n, uint64_t fo) {
+    const uint64_t E = dtype == JBO_F32 ? 4 : 8;
+    uint64_t sum = 0;
+    if (n == 0) return 0;
+    for (uint64_t v = fo / E; v <= (fo + n - 1) / E; ++v) {
+        uint32_t words[4] = {0, 0, 0, 0};
+        for (uint64_t t = 0; t < E; ++t) {
+            uint64_t e = v * E + t;
+            if (e < fo || e >= fo + n) continue;
+            uint64_t i = e - fo;
+            if (dtype == JBO_F32) {
+                uint32_t b;
+                memcpy(&b, (const float*)theta + i, 4);
+                words[t] = b;
+            } else {
+                uint32_t b = ((const uint16_t*)theta)[i];
+                words[t / 2] |= b << (16 * (t % 2));
+            }
+        }
+        sum += jbo_window_hash(v, words);
+    }
+    return sum;
+}
+
+/* ------------------------------------------------------------------------ */
 /* Threads                                                                    */
 /* ------------------------------------------------------------------------ */
 void jbo_set_threads(int n) {

@@ -53,6 +53,9 @@ int jbo_update_at(const void* in, void* out, int dtype, const uint64_t* idx, uin
 int jbo_update_delta_at(const uint64_t* idx, uint64_t n, const jbo_seed* seeds, const int8_t* q,
                         int K, double lr, double denom, double qscale, double* out);
 
+uint64_t jbo_window_hash(uint64_t window, const uint32_t words[4]);
+uint64_t jbo_checksum_segment(const void* theta, int dtype, uint64_t n, uint64_t fo);
+
 void jbo_set_threads(int n);
 int jbo_get_threads(void);
 

@@ -32,6 +32,7 @@ def aten_philox():
         os.replace(tmp, out)
     L = ctypes.CDLL(out)
     L.aten_philox_blocks.argtypes = [ctypes.c_uint64] * 4 + [ctypes.c_void_p]
+    L.aten_philox_rounds.argtypes = [ctypes.c_uint64] * 3 + [ctypes.c_int, ctypes.c_void_p]
     return L
 
 

@@ -13,3 +13,11 @@ extern "C" void aten_philox_blocks(uint64_t seed, uint64_t subsequence, uint64_t
         for (int w = 0; w < 4; ++w) out[4 * i + w] = engine();
     }
 }
+
+// The first `rounds` Philox rounds of counter (offset lo, offset hi, subsequence lo,
+// subsequence hi) under key `seed`: at::Philox4_32 takes the round count per draw.
+extern "C" void aten_philox_rounds(uint64_t seed, uint64_t subsequence, uint64_t offset,
+                                   int rounds, uint32_t* out) {
+    at::Philox4_32 engine(seed, subsequence, offset);
+    for (int w = 0; w < 4; ++w) out[w] = engine(rounds);
+}
