@@ -410,6 +410,7 @@ def run_sweep(a, jb, table, mids, stream):
                 "hbm_gbs": 2 * table.tensors[0].element_size() * N / (pms / 1e3) / 1e9})
     if a.next_legs:
         out.extend(next_legs(a, jb, table, stream))
+        out.append(checksum_leg(jb, table, stream))
     if a.sweep_out:
         with open(a.sweep_out, "w") as f:
             for ln in out:
@@ -470,6 +471,23 @@ def next_legs(a, jb, table, stream):
                         "ms": x0.elapsed_time(x1),
                         "param_seed_per_s": table.numel * T * Kt / (x0.elapsed_time(x1) / 1e3)})
     return out
+
+
+def checksum_leg(jb, table, stream):
+    """The model checksum (ChecksumMatch): one read of theta, HBM-bound."""
+    import torch
+    out = torch.zeros(1, dtype=torch.int64, device="cuda")
+    jb.jb_checksum(table, out, stream)
+    x0, x1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    reps = 5
+    x0.record(stream)
+    for _ in range(reps):
+        jb.jb_checksum(table, out, stream)
+    x1.record(stream)
+    torch.cuda.synchronize()
+    ms = x0.elapsed_time(x1) / reps
+    nbytes = table.numel * table.tensors[0].element_size()
+    return {"leg": "checksum", "ms": ms, "bytes": nbytes, "hbm_gbs": nbytes / (ms / 1e3) / 1e9}
 
 
 if __name__ == "__main__":

@@ -164,6 +164,23 @@ int jb_replay_updates(const jb_segment* segs, int n_segs, int dtype, const jb_se
                       const float* denom, float qscale, struct CUstream_st* stream);
 
 /*
+ * jb_checksum -- hash of the model for ChecksumMatch (Algorithm 1: each machine
+ * checks with a random peer that their hashed theta match). The paper fixes no
+ * hash. This one: cut the global element index space into 16-byte windows of
+ * storage (8 bf16 or 4 fp32 elements; window v = elements [vE, vE + E)). For
+ * every segment and every window v it overlaps, take the window's four 32-bit
+ * storage words (little-endian; elements outside the segment read as 0), apply
+ * the first four Philox4x32 rounds under key (lo32(v) ^ 0x6A09E667,
+ * hi32(v) ^ 0xF3BCC908), and add (x1:x0) + (x3:x2). The checksum is the sum
+ * mod 2^64. It depends on the values, the dtype and the flat offsets, not on
+ * the launch; replicas with the same table and bits get the same value.
+ *   d_out   device pointer to one uint64_t (8-byte aligned, caller-owned); it is
+ *           zeroed and written on `stream`.
+ */
+int jb_checksum(const jb_segment* segs, int n_segs, int dtype, uint64_t* d_out,
+                struct CUstream_st* stream);
+
+/*
  * jb_quantize_grad -- one-byte projected gradient (Section 3, Training
  * Speed: signed log of the gradient, clipped to +-127). Host only, pure:
  *   *out = sign(g) * min(127, round_half_away(qscale * ln(1 + |g|))),
@@ -202,8 +219,10 @@ int jb_debug_gaussian(jb_seed seed, uint64_t first_elem, uint64_t n, float* d_ou
 int jb_debug_box_muller(const uint32_t* d_words, uint64_t n_pairs, float* d_out,
                         struct CUstream_st* stream);
 
-/* jb_perturb / jb_apply_updates with an explicit number of CTAs (0 = the
- * default persistent grid); results must not depend on it. */
+/* jb_checksum / jb_perturb / jb_apply_updates with an explicit number of CTAs
+ * (0 = the default persistent grid); results must not depend on it. */
+int jb_checksum_with_grid(const jb_segment* segs, int n_segs, int dtype, uint64_t* d_out,
+                          int grid_ctas, struct CUstream_st* stream);
 int jb_perturb_with_grid(const jb_segment* segs, int n_segs, int dtype, jb_seed seed, float eps,
                          int grid_ctas, struct CUstream_st* stream);
 int jb_apply_updates_with_grid(const jb_segment* segs, int n_segs, int dtype,

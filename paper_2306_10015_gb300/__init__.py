@@ -10,6 +10,7 @@ streams. The functions keep the C names:
   restore of Algorithm 1 fused in
 * ``jb_replay_updates``  several steps' updates in one pass (a late joiner's
   catch-up, Appendix B)
+* ``jb_checksum``  the model hash of ChecksumMatch (Algorithm 1)
 * ``jb_quantize_grad`` / ``jb_dequantize_grad``  the one-byte projected
   gradient (Section 3, Training Speed)
 
@@ -74,6 +75,8 @@ def lib() -> ctypes.CDLL:
             L.jb_apply_updates_from.argtypes = [vp, vp, i32, i32, vp, vp, i32, f32, f32, f32,
                                                 i32, vp]
             L.jb_replay_updates.argtypes = [vp, i32, i32, vp, vp, vp, i32, vp, vp, f32, vp]
+            L.jb_checksum.argtypes = [vp, i32, i32, vp, vp]
+            L.jb_checksum_with_grid.argtypes = [vp, i32, i32, vp, i32, vp]
             L.jb_quantize_grad.argtypes = [ctypes.c_double, f32, ctypes.POINTER(ctypes.c_int8)]
             L.jb_dequantize_grad.argtypes = [ctypes.c_int8, f32, ctypes.POINTER(ctypes.c_float)]
             L.jb_max_seeds_per_call.argtypes = []
@@ -84,6 +87,7 @@ def lib() -> ctypes.CDLL:
             L.jb_debug_box_muller.argtypes = [vp, u64, vp, vp]
             for f in ("jb_perturb", "jb_perturb_with_grid", "jb_apply_updates",
                       "jb_apply_updates_with_grid", "jb_apply_updates_from", "jb_replay_updates",
+                      "jb_checksum", "jb_checksum_with_grid",
                       "jb_quantize_grad", "jb_dequantize_grad",
                       "jb_max_seeds_per_call", "jb_debug_philox", "jb_debug_gaussian",
                       "jb_debug_box_muller"):
@@ -245,6 +249,18 @@ def jb_replay_updates(table: ParamTable, steps, qscale: float, stream=None) -> N
                                    _stream(stream)))
 
 
+def jb_checksum(table: ParamTable, out, stream=None, grid_ctas: int = 0) -> None:
+    """out (CUDA int64 tensor, one element) <- the model checksum, on `stream`."""
+    L = lib()
+    if grid_ctas:
+        rc = L.jb_checksum_with_grid(table.segments, table.n_segments, table.dtype, out.data_ptr(),
+                                     int(grid_ctas), _stream(stream))
+    else:
+        rc = L.jb_checksum(table.segments, table.n_segments, table.dtype, out.data_ptr(),
+                           _stream(stream))
+    _check(rc)
+
+
 def jb_quantize_grad(g: float, qscale: float = 1.0) -> int:
     out = ctypes.c_int8()
     _check(lib().jb_quantize_grad(float(g), float(qscale), ctypes.byref(out)))
@@ -284,7 +300,7 @@ def jb_debug_box_muller(words, n_pairs: int, out, stream=None) -> None:
 __all__ = [
     "JB_OK", "JB_F32", "JB_BF16", "SEED_DTYPE", "JbError", "ParamTable", "jb_segment", "jb_seed",
     "lib", "seeds_array", "default_flat_offsets", "jb_perturb", "jb_apply_updates",
-    "jb_apply_updates_from", "jb_replay_updates",
+    "jb_apply_updates_from", "jb_replay_updates", "jb_checksum",
     "jb_quantize_grad", "jb_dequantize_grad", "jb_max_seeds_per_call", "jb_status_string",
     "jb_debug_philox", "jb_debug_gaussian", "jb_debug_box_muller",
 ]

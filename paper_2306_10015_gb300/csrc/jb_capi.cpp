@@ -356,6 +356,39 @@ JB_EXPORT int jb_apply_updates_with_grid(const jb_segment* segs, int n_segs, int
     return update_impl(segs, n_segs, dtype, seeds, q, K, lr, denom, qscale, grid_ctas, stream);
 }
 
+namespace {
+int checksum_impl(const jb_segment* segs, int n_segs, int dtype, uint64_t* d_out, int grid_ctas,
+                  cudaStream_t stream) {
+    std::vector<Seg> v;
+    int rc = collect_segments(segs, n_segs, dtype, v);
+    if (rc != JB_OK) return rc;
+    if (d_out == nullptr) return JB_ERR_INVALID_ARG;
+    if (reinterpret_cast<uint64_t>(d_out) & 7ull) return JB_ERR_MISALIGNED;
+    rc = cuda_status(cudaMemsetAsync(d_out, 0, sizeof(uint64_t), stream));
+    if (rc != JB_OK) return rc;
+    static thread_local jb::PerturbParams params;
+    params.n_seeds = 0;
+    for (size_t first = 0; first < v.size(); first += jb::kMaxSegsPerturb) {
+        const size_t count = std::min<size_t>(jb::kMaxSegsPerturb, v.size() - first);
+        pack_segments(v, first, count, dtype, params);
+        rc = cuda_status(jb::launch_checksum(params, dtype, reinterpret_cast<unsigned long long*>(d_out),
+                                             grid_ctas, stream));
+        if (rc != JB_OK) return rc;
+    }
+    return JB_OK;
+}
+}  // namespace
+
+JB_EXPORT int jb_checksum(const jb_segment* segs, int n_segs, int dtype, uint64_t* d_out,
+                          struct CUstream_st* stream) {
+    return checksum_impl(segs, n_segs, dtype, d_out, 0, stream);
+}
+
+JB_EXPORT int jb_checksum_with_grid(const jb_segment* segs, int n_segs, int dtype, uint64_t* d_out,
+                                    int grid_ctas, struct CUstream_st* stream) {
+    return checksum_impl(segs, n_segs, dtype, d_out, grid_ctas, stream);
+}
+
 JB_EXPORT int jb_quantize_grad(double g, float qscale, int8_t* out) {
     if (out == nullptr || !std::isfinite(qscale) || !(qscale > 0.0f)) return JB_ERR_INVALID_ARG;
     if (std::isnan(g)) {

@@ -84,6 +84,8 @@ enum DType { kF32 = 0, kBF16 = 1 };
 cudaError_t launch_update(const UpdateParams& p, int dtype, int grid_ctas, cudaStream_t s);
 cudaError_t launch_perturb(const PerturbParams& p, int dtype, int grid_ctas, cudaStream_t s);
 cudaError_t launch_general(const GeneralParams& p, int dtype, int grid_ctas, cudaStream_t s);
+cudaError_t launch_checksum(const PerturbParams& p, int dtype, unsigned long long* out,
+                            int grid_ctas, cudaStream_t s);
 cudaError_t launch_debug_philox(SeedParam seed, uint64_t first_block, uint64_t n_blocks,
                                 uint32_t* out, cudaStream_t s);
 cudaError_t launch_debug_gaussian(SeedParam seed, uint64_t first, uint64_t n, float* out,

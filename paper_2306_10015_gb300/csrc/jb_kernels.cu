@@ -6,6 +6,10 @@
 //                            theta_e <- round_T(theta_e + sum_k c_k z_e(s_k)),
 //                            the K pairs regenerated in registers, so theta is
 //                            read once and written once whatever K is.
+//   general_update_kernel<T> the update read from one table and written to
+//                            another, seeds in groups rounded to T after each
+//                            (the backup-fused restore and the multi-step replay).
+//   checksum_kernel<T>       the model checksum of ChecksumMatch (Algorithm 1).
 //   debug kernels            raw Philox words, z by element, Box-Muller of given
 //                            words (test hooks only).
 //
@@ -359,6 +363,98 @@ __global__ void __launch_bounds__(kThreads) general_update_kernel(const __grid_c
     }
 }
 
+// Model checksum (ChecksumMatch, Algorithm 1): the sum mod 2^64, over 16-byte
+// windows of the global element space, of four Philox rounds of the window's
+// storage words (elements outside the segment read as 0) keyed by the window
+// index; per window (x1:x0) + (x3:x2). Integer addition is order-free, so one
+// atomic add per CTA gives the same bits for any grid. Bound by HBM: one read
+// of theta, one wide multiply pair per window and round.
+constexpr uint32_t kSumKey0 = 0x6A09E667u, kSumKey1 = 0xF3BCC908u;
+constexpr int kSumRounds = 4;
+#ifndef JB_SUM_V
+#define JB_SUM_V 4
+#endif
+constexpr int kSumV = JB_SUM_V;  // 16-byte loads in flight per thread
+
+__device__ __forceinline__ uint64_t window_hash(uint64_t win, uint4 w) {
+    uint32_t x0 = w.x, x1 = w.y, x2 = w.z, x3 = w.w;
+    uint32_t k0 = static_cast<uint32_t>(win) ^ kSumKey0;
+    uint32_t k1 = static_cast<uint32_t>(win >> 32) ^ kSumKey1;
+#pragma unroll
+    for (int r = 0; r < kSumRounds; ++r) {
+        if (r > 0) {
+            k0 += kPhiloxW0;
+            k1 += kPhiloxW1;
+        }
+        philox_round(x0, x1, x2, x3, k0, k1);
+    }
+    return ((static_cast<uint64_t>(x1) << 32) | x0) + ((static_cast<uint64_t>(x3) << 32) | x2);
+}
+
+__device__ __forceinline__ uint32_t raw_bits(const float* p) { return __float_as_uint(*p); }
+__device__ __forceinline__ uint32_t raw_bits(const __nv_bfloat16* p) {
+    return *reinterpret_cast<const uint16_t*>(p);
+}
+
+template <typename T>
+__global__ void __launch_bounds__(kThreads) checksum_kernel(const __grid_constant__ PerturbParams p,
+                                                           unsigned long long* out) {
+    constexpr int E = Traits<T>::E;
+    constexpr int V = kSumV;
+    constexpr int BITS = 8 * static_cast<int>(sizeof(T));
+    const uint32_t lane = threadIdx.x & 31u;
+    const uint64_t warp = (static_cast<uint64_t>(blockIdx.x) * kThreads + threadIdx.x) >> 5;
+    const uint64_t n_warps = (static_cast<uint64_t>(gridDim.x) * kThreads) >> 5;
+    const uint64_t n_vec = p.n_vec;
+    const uint32_t n_segs = p.n_segs;
+    uint32_t s = 0;
+    uint64_t sum = 0;
+    for (uint64_t wt = warp; wt * (32u * V) < n_vec; wt += n_warps) {
+        uint4 w[V];
+        uint64_t win[V];
+        bool valid[V];
+#pragma unroll
+        for (int j = 0; j < V; ++j) {
+            const uint64_t vi = wt * (32u * V) + 32u * j + lane;
+            valid[j] = vi < n_vec;
+            if (valid[j])
+                while (s + 1 < n_segs && p.segs[s + 1].vec0 <= vi) ++s;
+            const SegParam& g = p.segs[s];
+            win[j] = g.fo / E + (vi - g.vec0);
+            const int64_t i0 = static_cast<int64_t>(win[j] * E) - static_cast<int64_t>(g.fo);
+            const int64_t n = static_cast<int64_t>(g.n);
+            const T* base = reinterpret_cast<const T*>(g.ptr & ~1ull);
+            if (valid[j] && (g.ptr & 1ull) && i0 >= 0 && i0 + E <= n) {
+                w[j] = __ldcs(reinterpret_cast<const uint4*>(base + i0));
+            } else {
+                uint32_t ww[4] = {0u, 0u, 0u, 0u};
+#pragma unroll
+                for (int t = 0; t < E; ++t) {
+                    const int64_t i = i0 + t;
+                    if (valid[j] && i >= 0 && i < n)
+                        ww[t * BITS / 32] |= raw_bits(base + i) << ((t * BITS) % 32);
+                }
+                w[j] = make_uint4(ww[0], ww[1], ww[2], ww[3]);
+            }
+        }
+#pragma unroll
+        for (int j = 0; j < V; ++j)
+            if (valid[j]) sum += window_hash(win[j], w[j]);
+    }
+    // CTA reduction; every thread reaches the barrier
+#pragma unroll
+    for (int d = 16; d > 0; d >>= 1) sum += __shfl_down_sync(0xFFFFFFFFu, sum, d);
+    __shared__ uint64_t part[kThreads / 32];
+    if (lane == 0) part[threadIdx.x >> 5] = sum;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        uint64_t t = 0;
+#pragma unroll
+        for (int i = 0; i < kThreads / 32; ++i) t += part[i];
+        atomicAdd(out, static_cast<unsigned long long>(t));
+    }
+}
+
 __global__ void debug_philox_kernel(SeedParam sp, uint64_t first, uint64_t n, uint32_t* out) {
     const uint64_t i = static_cast<uint64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
     if (i >= n) return;
@@ -396,7 +492,7 @@ __global__ void debug_box_muller_kernel(const uint32_t* words, uint64_t n, float
 
 // Persistent grid: SM count x resident CTAs per SM, cached per device and kernel.
 constexpr int kMaxDevices = 64;
-constexpr int kKernels = 6;
+constexpr int kKernels = 8;
 std::atomic<int> g_grid_cache[kMaxDevices][kKernels];
 
 template <typename K>
@@ -464,6 +560,29 @@ cudaError_t launch_general_t(const GeneralParams& p, int slot, int grid_ctas, cu
 cudaError_t launch_general(const GeneralParams& p, int dtype, int grid_ctas, cudaStream_t s) {
     if (dtype == kF32) return launch_general_t<float>(p, 4, grid_ctas, s);
     return launch_general_t<__nv_bfloat16>(p, 5, grid_ctas, s);
+}
+
+template <typename T>
+cudaError_t launch_checksum_t(const PerturbParams& p, unsigned long long* out, int slot,
+                              int grid_ctas, cudaStream_t stream) {
+    if (p.n_vec == 0) return cudaSuccess;
+    auto kernel = checksum_kernel<T>;
+    int grid = grid_ctas;
+    if (grid <= 0) {
+        cudaError_t err = persistent_grid(kernel, slot, &grid);
+        if (err != cudaSuccess) return err;
+        constexpr uint64_t vec_per_cta = 32ull * kSumV * (kThreads / 32);
+        const uint64_t needed = (p.n_vec + vec_per_cta - 1) / vec_per_cta;
+        if (needed < static_cast<uint64_t>(grid)) grid = static_cast<int>(needed);
+    }
+    kernel<<<grid, kThreads, 0, stream>>>(p, out);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_checksum(const PerturbParams& p, int dtype, unsigned long long* out,
+                            int grid_ctas, cudaStream_t s) {
+    if (dtype == kF32) return launch_checksum_t<float>(p, out, 6, grid_ctas, s);
+    return launch_checksum_t<__nv_bfloat16>(p, out, 7, grid_ctas, s);
 }
 
 cudaError_t launch_perturb(const PerturbParams& p, int dtype, int grid_ctas, cudaStream_t s) {

@@ -193,3 +193,12 @@ def test_apply_from_and_replay_validation(jb):
     assert replay(big, np.ones(2, np.float32)) == E["many"]                # one step > 512 pairs
     # two equal seeds in different steps are legal (only a step must be duplicate-free):
     # validation passes and the call reaches the launch, which has no device here
+
+
+def test_checksum_validation(jb):
+    import ctypes as C
+    src = _segs(jb, [(FAKE, 100, 0)])
+    L = jb.lib()
+    assert L.jb_checksum(src, 1, 0, None, None) == -1
+    assert L.jb_checksum(src, 1, 0, C.c_void_p(FAKE + 4), None) == -3
+    assert L.jb_checksum(src, 1, 3, C.c_void_p(FAKE), None) == -2
