@@ -93,6 +93,11 @@ def lib() -> ctypes.CDLL:
             L.jbo_update_delta_at.argtypes = [vp, u64, vp, vp, ctypes.c_int, ctypes.c_double,
                                               ctypes.c_double, ctypes.c_double, vp]
             L.jbo_update_delta_at.restype = ctypes.c_int
+            L.jbo_q4_levels.argtypes = [vp]
+            L.jbo_q4_quantize.argtypes = [vp, u64, vp, vp]
+            L.jbo_q4_dequantize.argtypes = [vp, vp, u64, vp]
+            L.jbo_q4_perturb.argtypes = [vp, vp, u64, u64, _Seed, ctypes.c_double, vp]
+            L.jbo_q4_perturb.restype = ctypes.c_int
             L.jbo_window_hash.argtypes = [u64, u32p]
             L.jbo_window_hash.restype = ctypes.c_uint64
             L.jbo_checksum_segment.argtypes = [vp, ctypes.c_int, u64, u64]
@@ -271,6 +276,40 @@ def update_delta_at(idx: np.ndarray, seeds, q, lr: float, denom: float,
     _check(lib().jbo_update_delta_at(_ptr(i), i.size, _ptr(s), _ptr(qa), len(s), lr, denom,
                                      qscale, _ptr(out)))
     return out
+
+
+# --- 4-bit weights -----------------------------------------------------------
+
+def q4_levels() -> np.ndarray:
+    out = np.empty(16, dtype=np.float32)
+    lib().jbo_q4_levels(_ptr(out))
+    return out
+
+
+def q4_quantize(w) -> tuple:
+    """(codes uint8[(n + 1) // 2], scales float32[ceil(n / 64)]) of values w."""
+    w = np.ascontiguousarray(w, dtype=np.float64)
+    codes = np.zeros((w.size + 1) // 2, dtype=np.uint8)
+    scale = np.zeros((w.size + 63) // 64, dtype=np.float32)
+    lib().jbo_q4_quantize(_ptr(w), w.size, _ptr(codes), _ptr(scale))
+    return codes, scale
+
+
+def q4_dequantize(codes, scale, n: int) -> np.ndarray:
+    codes = np.ascontiguousarray(codes, dtype=np.uint8)
+    scale = np.ascontiguousarray(scale, dtype=np.float32)
+    w = np.empty(n, dtype=np.float64)
+    lib().jbo_q4_dequantize(_ptr(codes), _ptr(scale), n, _ptr(w))
+    return w
+
+
+def q4_perturb(codes, scale, n: int, flat_offset: int, seed, eps: float):
+    """(codes', scales', perturbed values before quantization) of one 4-bit tensor."""
+    c = np.array(codes, dtype=np.uint8, copy=True)
+    s = np.array(scale, dtype=np.float32, copy=True)
+    w = np.empty(n, dtype=np.float64)
+    _check(lib().jbo_q4_perturb(_ptr(c), _ptr(s), n, flat_offset, _seed(seed), eps, _ptr(w)))
+    return c, s, w
 
 
 # --- model checksum ----------------------------------------------------------

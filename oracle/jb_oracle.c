@@ -322,6 +322,89 @@ int jbo_update_delta_at(const uint64_t* idx, uint64_t n, const jbo_seed* seeds, 
 }
 
 /* ------------------------------------------------------------------------ */
+/* 4-bit weights (Section 3, Training Speed: weights are dequantized before   */
+/* the noise is added and quantized again). Reading (the paper fixes no       */
+/* format; it cites QLoRA's NormalFloat): 16 levels built from quantiles of   */
+/* N(0,1), 8 at probabilities delta + (1/2 - delta) j/7 (j = 0..7, the last   */
+/* is the median 0) and 8 more at 1/2 + (1/2 - delta) j/8 (j = 1..8), divided */
+/* by the largest so they span [-1, 1]; delta = 1/32. Levels are stored as    */
+/* fp32. Blocks of 64 elements share one fp32 scale, the largest |w| of the   */
+/* block; code = number of midpoints between adjacent levels lying strictly   */
+/* below w / scale (the nearest level, ties to the lower). Element 2i sits in */
+/* the low nibble of byte i.                                                  */
+/* ------------------------------------------------------------------------ */
+static double std_normal_quantile(double p) {
+    /* bisection on Phi(x) = erfc(-x / sqrt 2) / 2, to double precision */
+    double lo = -40.0, hi = 40.0;
+    for (int it = 0; it < 200; ++it) {
+        double mid = 0.5 * (lo + hi);
+        double phi = 0.5 * erfc(-mid / sqrt(2.0));
+        if (phi < p) lo = mid; else hi = mid;
+    }
+    return 0.5 * (lo + hi);
+}
+
+void jbo_q4_levels(float out[16]) {
+    const double delta = 1.0 / 32.0;
+    double v[16];
+    for (int j = 0; j < 8; ++j) v[j] = std_normal_quantile(delta + (0.5 - delta) * j / 7.0);
+    v[7] = 0.0;
+    for (int j = 1; j <= 8; ++j) v[7 + j] = std_normal_quantile(0.5 + (0.5 - delta) * j / 8.0);
+    double top = v[15];
+    for (int j = 0; j < 16; ++j) out[j] = (float)(v[j] / top);
+    out[7] = 0.0f;
+    out[15] = 1.0f;
+}
+
+static unsigned q4_code(double x, const float lev[16]) {
+    unsigned c = 0;
+    for (int j = 0; j < 15; ++j)
+        if (x > 0.5 * ((double)lev[j] + (double)lev[j + 1])) c = (unsigned)j + 1;
+    return c;
+}
+
+/* Quantize n values (a tensor) into codes (n + 1) / 2 bytes and scales per 64. */
+void jbo_q4_quantize(const double* w, uint64_t n, uint8_t* codes, float* scale) {
+    float lev[16];
+    jbo_q4_levels(lev);
+    for (uint64_t b = 0; b * 64 < n; ++b) {
+        uint64_t end = (b + 1) * 64 < n ? (b + 1) * 64 : n;
+        double m = 0.0;
+        for (uint64_t i = b * 64; i < end; ++i) if (fabs(w[i]) > m) m = fabs(w[i]);
+        scale[b] = (float)m;
+        for (uint64_t i = b * 64; i < end; ++i) {
+            unsigned c = q4_code(m > 0.0 ? w[i] / (double)scale[b] : 0.0, lev);
+            if (i % 2 == 0) codes[i / 2] = (uint8_t)((codes[i / 2] & 0xF0u) | c);
+            else codes[i / 2] = (uint8_t)((codes[i / 2] & 0x0Fu) | (c << 4));
+        }
+    }
+}
+
+void jbo_q4_dequantize(const uint8_t* codes, const float* scale, uint64_t n, double* w) {
+    float lev[16];
+    jbo_q4_levels(lev);
+    for (uint64_t i = 0; i < n; ++i) {
+        unsigned c = (i % 2 == 0) ? (codes[i / 2] & 0x0Fu) : (codes[i / 2] >> 4);
+        w[i] = (double)lev[c] * (double)scale[i / 64];
+    }
+}
+
+/* PerturbParameters on 4-bit weights: dequantize, add eps z, quantize again.
+ * Also returns the perturbed values before quantization in w_out (may be NULL). */
+int jbo_q4_perturb(uint8_t* codes, float* scale, uint64_t n, uint64_t flat_offset, jbo_seed s,
+                   double eps, double* w_out) {
+    double* w = (double*)malloc(sizeof(double) * (size_t)(n > 0 ? n : 1));
+    if (!w) return -2;
+    jbo_q4_dequantize(codes, scale, n, w);
+    #pragma omp parallel for schedule(static)
+    for (int64_t i = 0; i < (int64_t)n; ++i) w[i] += eps * jbo_gaussian(s, flat_offset + (uint64_t)i);
+    jbo_q4_quantize(w, n, codes, scale);
+    if (w_out) memcpy(w_out, w, sizeof(double) * (size_t)n);
+    free(w);
+    return 0;
+}
+
+/* ------------------------------------------------------------------------ */
 /* Model checksum for ChecksumMatch (Algorithm 1: "check if hashed theta      */
 /* matches peer's"). The paper fixes no hash. Reading: the global element     */
 /* index space is cut into windows of 16 bytes of storage (8 bf16 or 4 fp32   */

@@ -53,6 +53,12 @@ int jbo_update_at(const void* in, void* out, int dtype, const uint64_t* idx, uin
 int jbo_update_delta_at(const uint64_t* idx, uint64_t n, const jbo_seed* seeds, const int8_t* q,
                         int K, double lr, double denom, double qscale, double* out);
 
+void jbo_q4_levels(float out[16]);
+void jbo_q4_quantize(const double* w, uint64_t n, uint8_t* codes, float* scale);
+void jbo_q4_dequantize(const uint8_t* codes, const float* scale, uint64_t n, double* w);
+int jbo_q4_perturb(uint8_t* codes, float* scale, uint64_t n, uint64_t flat_offset, jbo_seed s,
+                   double eps, double* w_out);
+
 uint64_t jbo_window_hash(uint64_t window, const uint32_t words[4]);
 uint64_t jbo_checksum_segment(const void* theta, int dtype, uint64_t n, uint64_t fo);
 
