@@ -411,6 +411,7 @@ def run_sweep(a, jb, table, mids, stream):
     if a.next_legs:
         out.extend(next_legs(a, jb, table, stream))
         out.append(checksum_leg(jb, table, stream))
+        out.append(q4_leg(a, jb, stream))
     if a.sweep_out:
         with open(a.sweep_out, "w") as f:
             for ln in out:
@@ -488,6 +489,38 @@ def checksum_leg(jb, table, stream):
     ms = x0.elapsed_time(x1) / reps
     nbytes = table.numel * table.tensors[0].element_size()
     return {"leg": "checksum", "ms": ms, "bytes": nbytes, "hbm_gbs": nbytes / (ms / 1e3) / 1e9}
+
+
+def q4_leg(a, jb, stream):
+    """PerturbParameters on the benchmark's set stored as 4-bit weights (codes and
+    64-element scales, synthetic values), one pass read + write."""
+    import torch
+    import synthetic
+    specs = synthetic.opt_tensors(a.model)
+    g = torch.Generator(device="cuda")
+    g.manual_seed(synthetic.MASTER_SEED)
+    tensors = []
+    for sp in specs:
+        n = sp.numel
+        codes = torch.randint(0, 256, ((n + 1) // 2 + 8,), dtype=torch.uint8, device="cuda",
+                              generator=g)
+        scale = torch.rand(((n + 63) // 64,), device="cuda", generator=g) * 0.05
+        tensors.append((codes, scale, n))
+    table = jb.Q4Table(tensors)
+    jb.jb_perturb_q4(table, (1, 2, 3), a.eps, stream)
+    x0, x1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    x0.record(stream)
+    for i in range(3):
+        jb.jb_perturb_q4(table, (1, 2, 3), a.eps if i % 2 == 0 else -a.eps, stream)
+    x1.record(stream)
+    torch.cuda.synchronize()
+    ms = x0.elapsed_time(x1) / 3
+    n = sum(sp.numel for sp in specs)
+    nbytes = 2 * sum((sp.numel + 1) // 2 + 4 * ((sp.numel + 63) // 64) for sp in specs)
+    del tensors, table
+    torch.cuda.empty_cache()
+    return {"leg": "perturb_q4", "ms": ms, "param_seed_per_s": n / (ms / 1e3),
+            "hbm_gbs": nbytes / (ms / 1e3) / 1e9}
 
 
 if __name__ == "__main__":

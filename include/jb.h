@@ -163,6 +163,38 @@ int jb_replay_updates(const jb_segment* segs, int n_segs, int dtype, const jb_se
                       const int8_t* q, const int* step_sizes, int n_steps, const float* lr,
                       const float* denom, float qscale, struct CUstream_st* stream);
 
+/* A tensor of 4-bit weights: numel codes, two per byte (element 2i in the low
+ * nibble of byte i; `codes` 8-byte aligned, (numel + 1) / 2 bytes), and one fp32
+ * scale per block of 64 elements (`scale`, ceil(numel / 64) floats). Weight i
+ * is level[code_i] * scale[i / 64] with the 16 levels of jb_q4_levels().
+ * flat_offset (a multiple of 4) is the global index of element 0, as for
+ * jb_segment. Device memory, caller-owned. */
+typedef struct {
+    uint8_t* codes;
+    float* scale;
+    uint64_t numel;
+    uint64_t flat_offset;
+} jb_q4_segment;
+
+/*
+ * jb_perturb_q4 -- PerturbParameters on 4-bit weights (Section 3, Training
+ * Speed: weights are dequantized before the noise is added and quantized
+ * again). For every block of 64 elements: w_i = level[code_i] * scale,
+ * w'_i = fma(eps, z_i(seed), w_i) in fp32 with the same z as jb_perturb, then
+ * scale' = max_i |w'_i| and code'_i = the nearest level to w'_i / scale' (ties
+ * to the lower level; scale' = 0 gives the zero level). Codes and scales are
+ * rewritten in place, asynchronously on `stream`. The paper fixes no 4-bit
+ * format; this is a NormalFloat-style code after QLoRA (see jb_q4_levels).
+ */
+int jb_perturb_q4(const jb_q4_segment* segs, int n_segs, jb_seed seed, float eps,
+                  struct CUstream_st* stream);
+
+/* The 16 levels of the 4-bit code, ascending, in [-1, 1]: quantiles of N(0,1)
+ * at probabilities d + (1/2 - d) j / 7 (j = 0..7, the median 0 last) and
+ * 1/2 + (1/2 - d) j / 8 (j = 1..8), d = 1/32, divided by the largest, rounded
+ * to fp32. Host only; out receives 16 floats. */
+int jb_q4_levels(float* out);
+
 /*
  * jb_checksum -- hash of the model for ChecksumMatch (Algorithm 1: each machine
  * checks with a random peer that their hashed theta match). The paper fixes no

@@ -11,6 +11,7 @@ streams. The functions keep the C names:
 * ``jb_replay_updates``  several steps' updates in one pass (a late joiner's
   catch-up, Appendix B)
 * ``jb_checksum``  the model hash of ChecksumMatch (Algorithm 1)
+* ``jb_perturb_q4``  the perturbation of 4-bit weights (Section 3)
 * ``jb_quantize_grad`` / ``jb_dequantize_grad``  the one-byte projected
   gradient (Section 3, Training Speed)
 
@@ -47,6 +48,11 @@ class jb_segment(ctypes.Structure):
                 ("flat_offset", ctypes.c_uint64)]
 
 
+class jb_q4_segment(ctypes.Structure):
+    _fields_ = [("codes", ctypes.c_void_p), ("scale", ctypes.c_void_p), ("numel", ctypes.c_uint64),
+                ("flat_offset", ctypes.c_uint64)]
+
+
 class jb_seed(ctypes.Structure):
     _fields_ = [("machine_id", ctypes.c_uint64), ("step", ctypes.c_uint32),
                 ("sample_id", ctypes.c_uint32)]
@@ -75,6 +81,8 @@ def lib() -> ctypes.CDLL:
             L.jb_apply_updates_from.argtypes = [vp, vp, i32, i32, vp, vp, i32, f32, f32, f32,
                                                 i32, vp]
             L.jb_replay_updates.argtypes = [vp, i32, i32, vp, vp, vp, i32, vp, vp, f32, vp]
+            L.jb_perturb_q4.argtypes = [vp, i32, jb_seed, f32, vp]
+            L.jb_q4_levels.argtypes = [vp]
             L.jb_checksum.argtypes = [vp, i32, i32, vp, vp]
             L.jb_checksum_with_grid.argtypes = [vp, i32, i32, vp, i32, vp]
             L.jb_quantize_grad.argtypes = [ctypes.c_double, f32, ctypes.POINTER(ctypes.c_int8)]
@@ -87,7 +95,7 @@ def lib() -> ctypes.CDLL:
             L.jb_debug_box_muller.argtypes = [vp, u64, vp, vp]
             for f in ("jb_perturb", "jb_perturb_with_grid", "jb_apply_updates",
                       "jb_apply_updates_with_grid", "jb_apply_updates_from", "jb_replay_updates",
-                      "jb_checksum", "jb_checksum_with_grid",
+                      "jb_checksum", "jb_checksum_with_grid", "jb_perturb_q4", "jb_q4_levels",
                       "jb_quantize_grad", "jb_dequantize_grad",
                       "jb_max_seeds_per_call", "jb_debug_philox", "jb_debug_gaussian",
                       "jb_debug_box_muller"):
@@ -249,6 +257,36 @@ def jb_replay_updates(table: ParamTable, steps, qscale: float, stream=None) -> N
                                    _stream(stream)))
 
 
+class Q4Table:
+    """jb_q4_segment array over 4-bit tensors: (codes uint8 CUDA tensor, scales float32 CUDA
+    tensor, numel) triples; flat offsets default to the jb_segment rule."""
+
+    def __init__(self, tensors, flat_offsets: Optional[Sequence[int]] = None):
+        self.tensors = list(tensors)
+        numels = [int(n) for _, _, n in self.tensors]
+        self.flat_offsets = (list(flat_offsets) if flat_offsets is not None
+                             else default_flat_offsets(numels))
+        n = len(self.tensors)
+        self.segments = (jb_q4_segment * n)()
+        for i, ((codes, scale, numel), fo) in enumerate(zip(self.tensors, self.flat_offsets)):
+            if codes.numel() < (numel + 1) // 2 or scale.numel() < (numel + 63) // 64:
+                raise ValueError("codes or scales too short for numel")
+            self.segments[i] = jb_q4_segment(codes.data_ptr(), scale.data_ptr(), int(numel), int(fo))
+        self.n_segments = n
+
+
+def jb_perturb_q4(table: "Q4Table", seed, eps: float, stream=None) -> None:
+    """4-bit weights: dequantize, add eps z(seed), quantize again, in place."""
+    _check(lib().jb_perturb_q4(table.segments, table.n_segments, _seed(seed), float(eps),
+                               _stream(stream)))
+
+
+def jb_q4_levels() -> np.ndarray:
+    out = np.empty(16, dtype=np.float32)
+    _check(lib().jb_q4_levels(out.ctypes.data))
+    return out
+
+
 def jb_checksum(table: ParamTable, out, stream=None, grid_ctas: int = 0) -> None:
     """out (CUDA int64 tensor, one element) <- the model checksum, on `stream`."""
     L = lib()
@@ -300,7 +338,8 @@ def jb_debug_box_muller(words, n_pairs: int, out, stream=None) -> None:
 __all__ = [
     "JB_OK", "JB_F32", "JB_BF16", "SEED_DTYPE", "JbError", "ParamTable", "jb_segment", "jb_seed",
     "lib", "seeds_array", "default_flat_offsets", "jb_perturb", "jb_apply_updates",
-    "jb_apply_updates_from", "jb_replay_updates", "jb_checksum",
+    "jb_apply_updates_from", "jb_replay_updates", "jb_checksum", "jb_perturb_q4", "jb_q4_levels",
+    "Q4Table", "jb_q4_segment",
     "jb_quantize_grad", "jb_dequantize_grad", "jb_max_seeds_per_call", "jb_status_string",
     "jb_debug_philox", "jb_debug_gaussian", "jb_debug_box_muller",
 ]

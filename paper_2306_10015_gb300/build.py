@@ -20,7 +20,7 @@ OUT_DIR = os.path.join(PKG, "_build")
 LIB = os.path.join(OUT_DIR, "libjb.so")
 
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
-SOURCES = ["jb_kernels.cu", "jb_capi.cpp"]
+SOURCES = ["jb_kernels.cu", "jb_q4.cu", "jb_capi.cpp"]
 HEADERS = ["jb_rng.cuh", "jb_internal.h"]
 
 

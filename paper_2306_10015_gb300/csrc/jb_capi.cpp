@@ -389,6 +389,63 @@ JB_EXPORT int jb_checksum_with_grid(const jb_segment* segs, int n_segs, int dtyp
     return checksum_impl(segs, n_segs, dtype, d_out, grid_ctas, stream);
 }
 
+JB_EXPORT int jb_perturb_q4(const jb_q4_segment* segs, int n_segs, jb_seed seed, float eps,
+                            struct CUstream_st* stream) {
+    if (n_segs < 0 || (n_segs > 0 && segs == nullptr)) return JB_ERR_INVALID_ARG;
+    if (!std::isfinite(eps)) return JB_ERR_INVALID_ARG;
+    struct Q { uint64_t codes, scale, fo, n; };
+    std::vector<Q> v;
+    struct Iv { uint64_t a, b; };
+    std::vector<Iv> mem, idx;
+    for (int i = 0; i < n_segs; ++i) {
+        const jb_q4_segment& g = segs[i];
+        if (g.numel == 0) continue;
+        const uint64_t c = reinterpret_cast<uint64_t>(g.codes), sp = reinterpret_cast<uint64_t>(g.scale);
+        if (c == 0 || sp == 0) return JB_ERR_INVALID_ARG;
+        if ((c & 7ull) || (sp & 3ull) || (g.flat_offset & 3ull)) return JB_ERR_MISALIGNED;
+        if (g.numel > kMaxIndex || g.flat_offset > kMaxIndex - g.numel) return JB_ERR_INVALID_ARG;
+        const uint64_t nb = (g.numel + 1) / 2, ns = 4 * ((g.numel + 63) / 64);
+        if (c > UINT64_MAX - nb || sp > UINT64_MAX - ns) return JB_ERR_INVALID_ARG;
+        v.push_back({c, sp, g.flat_offset, g.numel});
+        mem.push_back({c, c + nb});
+        mem.push_back({sp, sp + ns});
+        idx.push_back({g.flat_offset, g.flat_offset + g.numel});
+    }
+    for (auto* list : {&mem, &idx}) {
+        std::sort(list->begin(), list->end(), [](const Iv& x, const Iv& y) { return x.a < y.a; });
+        for (size_t i = 1; i < list->size(); ++i)
+            if ((*list)[i - 1].b > (*list)[i].a) return JB_ERR_INVALID_ARG;
+    }
+    if (v.empty()) return JB_OK;
+    static thread_local jb::Q4Params params;
+    params.seed = seed_param(seed, eps);
+    for (size_t first = 0; first < v.size(); first += jb::kMaxSegsQ4) {
+        const size_t count = std::min<size_t>(jb::kMaxSegsQ4, v.size() - first);
+        uint64_t unit = 0;
+        for (size_t i = 0; i < count; ++i) {
+            const Q& q = v[first + i];
+            jb::SegParamQ4& g = params.segs[i];
+            g.codes = q.codes;
+            g.scale = q.scale;
+            g.fo = q.fo;
+            g.n = q.n;
+            g.unit0 = unit;
+            unit += 4 * ((q.n + 63) / 64);  // whole 64-element blocks of 16-element units
+        }
+        params.n_segs = static_cast<uint32_t>(count);
+        params.n_units = unit;
+        const int rc = cuda_status(jb::launch_q4_perturb(params, 0, stream));
+        if (rc != JB_OK) return rc;
+    }
+    return JB_OK;
+}
+
+JB_EXPORT int jb_q4_levels(float* out) {
+    if (out == nullptr) return JB_ERR_INVALID_ARG;
+    jb::q4_levels_host(out);
+    return JB_OK;
+}
+
 JB_EXPORT int jb_quantize_grad(double g, float qscale, int8_t* out) {
     if (out == nullptr || !std::isfinite(qscale) || !(qscale > 0.0f)) return JB_ERR_INVALID_ARG;
     if (std::isnan(g)) {

@@ -78,6 +78,32 @@ struct GeneralParams {
 
 static_assert(sizeof(GeneralParams) <= 32764, "general launch exceeds the parameter space");
 
+// 4-bit weights: codes (two per byte, element 2i in the low nibble) and one fp32
+// scale per 64 elements. Work unit: 16 elements (8 code bytes); a segment owns
+// units [unit0, unit0 + ceil(n / 64) * 4), so a 64-element block is always four
+// consecutive units, handled by four consecutive lanes.
+constexpr int kMaxSegsQ4 = 800;
+
+struct SegParamQ4 {
+    uint64_t codes;  // device address, 8-byte aligned
+    uint64_t scale;  // device address of the fp32 scales
+    uint64_t fo;     // global index of element 0 (a multiple of 4)
+    uint64_t n;
+    uint64_t unit0;
+};
+
+struct Q4Params {
+    SeedParam seed;  // coef = eps
+    uint32_t n_segs;
+    uint64_t n_units;
+    SegParamQ4 segs[kMaxSegsQ4];
+};
+
+static_assert(sizeof(Q4Params) <= 32764, "4-bit launch exceeds the parameter space");
+
+cudaError_t launch_q4_perturb(const Q4Params& p, int grid_ctas, cudaStream_t s);
+void q4_levels_host(float out[16]);
+
 enum DType { kF32 = 0, kBF16 = 1 };
 
 // Launchers (jb_kernels.cu). grid_ctas <= 0 selects the persistent grid.

@@ -1,0 +1,176 @@
+// jb_q4.cu -- PerturbParameters on 4-bit weights (Section 3, Training Speed:
+// layer weights are dequantized before the noise is added and quantized again).
+//
+// Code (the paper fixes none; it cites QLoRA's NormalFloat): 16 levels built
+// from quantiles of N(0,1) and scaled to [-1, 1] (gen_q4_levels.py); blocks of
+// 64 elements share one fp32 scale, the largest |w| of the block; a weight is
+// level[code] * scale; quantizing picks the nearest level (ties to the lower).
+//
+// Per element: dequantize, w' = fma(eps, z, w) with the same z as every other
+// path (global index flat_offset + i), then per block scale' = max |w'| and
+// code' = nearest level of w' / scale'. Codes and scales are rewritten in place.
+// A 64-element block is four consecutive lanes (16 elements each): its maximum
+// is two butterfly shuffles. Levels and midpoints live in shared memory, read
+// with data-dependent indices (16 distinct words: no bank conflicts).
+#include <cuda_bf16.h>
+
+#include <atomic>
+
+#include "jb_internal.h"
+#include "jb_rng.cuh"
+
+namespace jb {
+namespace {
+
+// gen_q4_levels.py
+constexpr float kQ4Level[16] = {
+    -0x1.000000p+0f, -0x1.6311acp-1f, -0x1.0b8d60p-1f, -0x1.924c0ap-2f, -0x1.21b102p-2f,
+    -0x1.7851c6p-3f, -0x1.72d976p-4f, 0x0.0p+0f,       0x1.4421acp-4f,  0x1.47c076p-3f,
+    0x1.f54804p-3f,  0x1.582f80p-2f,  0x1.c1002ap-2f,  0x1.1eba52p-1f,  0x1.70ca9ap-1f,
+    0x1.000000p+0f};
+
+__constant__ float c_level[16] = {
+    kQ4Level[0], kQ4Level[1], kQ4Level[2],  kQ4Level[3],  kQ4Level[4],  kQ4Level[5],
+    kQ4Level[6], kQ4Level[7], kQ4Level[8],  kQ4Level[9],  kQ4Level[10], kQ4Level[11],
+    kQ4Level[12], kQ4Level[13], kQ4Level[14], kQ4Level[15]};
+// midpoints (L_j + L_j+1) / 2 of the fp32 levels, rounded to fp32 (gen_q4_levels.py)
+__constant__ float c_mid[15] = {
+    -0x1.b188d6p-1f, -0x1.374f86p-1f, -0x1.d4b364p-2f, -0x1.59fe86p-2f, -0x1.ddd9e4p-3f,
+    -0x1.18df40p-3f, -0x1.72d976p-5f, 0x1.4421acp-5f,  0x1.e9d14cp-4f,  0x1.9e843cp-3f,
+    0x1.2969c0p-2f,  0x1.8c97d4p-2f,  0x1.ff3a68p-2f,  0x1.47c276p-1f,  0x1.b8654cp-1f};
+
+// Nearest level of x: the number of midpoints strictly below x, by binary search.
+__device__ __forceinline__ uint32_t q4_code(float x, const float* mid) {
+    uint32_t c = 0;
+    if (x > mid[c + 7]) c += 8;
+    if (x > mid[c + 3]) c += 4;
+    if (x > mid[c + 1]) c += 2;
+    if (x > mid[c + 0]) c += 1;
+    return c;
+}
+
+constexpr int kThreadsQ4 = 256;
+
+__global__ void __launch_bounds__(kThreadsQ4) q4_perturb_kernel(const __grid_constant__ Q4Params p) {
+    __shared__ float level[16];
+    __shared__ float mid[16];
+    if (threadIdx.x < 16) {
+        level[threadIdx.x] = c_level[threadIdx.x];
+        mid[threadIdx.x] = threadIdx.x < 15 ? c_mid[threadIdx.x] : 2.0f;
+    }
+    __syncthreads();  // every thread reaches this before any work
+
+    const uint32_t lane = threadIdx.x & 31u;
+    const uint64_t warp = (static_cast<uint64_t>(blockIdx.x) * kThreadsQ4 + threadIdx.x) >> 5;
+    const uint64_t n_warps = (static_cast<uint64_t>(gridDim.x) * kThreadsQ4) >> 5;
+    const SeedConst sc = seed_const(Key{p.seed.k0, p.seed.k1, p.seed.step, p.seed.sample});
+    const float eps = p.seed.coef;
+    uint32_t s = 0;
+    // all 32 lanes run every iteration (the block maximum is a warp shuffle)
+    for (uint64_t wt = warp; wt * 32u < p.n_units; wt += n_warps) {
+        const uint64_t unit = wt * 32u + lane;
+        const bool valid = unit < p.n_units;
+        if (valid)
+            while (s + 1 < p.n_segs && p.segs[s + 1].unit0 <= unit) ++s;
+        const SegParamQ4& g = p.segs[s];
+        const uint64_t u = unit - g.unit0;
+        const int64_t i0 = static_cast<int64_t>(16 * u);
+        const int64_t n = static_cast<int64_t>(g.n);
+        const bool any = valid && i0 < n;
+        const bool full = valid && i0 + 16 <= n;
+        uint8_t* codes = reinterpret_cast<uint8_t*>(g.codes);
+        float* scale = reinterpret_cast<float*>(g.scale);
+
+        uint32_t cw[2] = {0u, 0u};  // 16 codes
+        if (full) {
+            const uint2 v = *reinterpret_cast<const uint2*>(codes + i0 / 2);
+            cw[0] = v.x;
+            cw[1] = v.y;
+        } else if (any) {
+#pragma unroll
+            for (int b = 0; b < 8; ++b)
+                if (i0 + 2 * b < n) cw[b / 4] |= static_cast<uint32_t>(codes[i0 / 2 + b]) << (8 * (b % 4));
+        }
+        const float sc_in = any ? scale[u >> 2] : 0.0f;
+
+        // dequantize and perturb
+        float w[16];
+        uint4 words[4];
+        const uint64_t blk0 = (g.fo + static_cast<uint64_t>(i0)) >> 2;  // fo % 4 == 0
+#pragma unroll
+        for (int b = 0; b < 4; ++b)
+            words[b] = philox_block(sc, static_cast<uint32_t>(blk0 + b),
+                                    static_cast<uint32_t>((blk0 + b) >> 32));
+        float m = 0.0f;
+#pragma unroll
+        for (int b = 0; b < 4; ++b) {
+            const GaussPair z = box_muller2(words[b]);
+            const float zz[4] = {z.even.x, z.odd.x, z.even.y, z.odd.y};
+#pragma unroll
+            for (int t = 0; t < 4; ++t) {
+                const int k = 4 * b + t;
+                const uint32_t c = (cw[k / 8] >> (4 * (k % 8))) & 0xFu;
+                const float v = __fmaf_rn(eps, zz[t], __fmul_rn(level[c], sc_in));
+                w[k] = v;
+                if (i0 + k < n) m = fmaxf(m, fabsf(v));
+            }
+        }
+        // block maximum over the four lanes of the block (lanes 4j .. 4j + 3)
+        m = fmaxf(m, __shfl_xor_sync(0xFFFFFFFFu, m, 1));
+        m = fmaxf(m, __shfl_xor_sync(0xFFFFFFFFu, m, 2));
+        const float inv = m > 0.0f ? __frcp_rn(m) : 0.0f;
+
+        // quantize again
+        uint32_t ow[2] = {0u, 0u};
+#pragma unroll
+        for (int k = 0; k < 16; ++k) ow[k / 8] |= q4_code(__fmul_rn(w[k], inv), mid) << (4 * (k % 8));
+        if (full) {
+            *reinterpret_cast<uint2*>(codes + i0 / 2) = make_uint2(ow[0], ow[1]);
+        } else if (any) {
+#pragma unroll
+            for (int b = 0; b < 8; ++b) {
+                if (i0 + 2 * b >= n) continue;
+                const uint8_t byte = static_cast<uint8_t>(ow[b / 4] >> (8 * (b % 4)));
+                // an odd tail leaves the unused high nibble of the last byte as it was
+                codes[i0 / 2 + b] = (i0 + 2 * b + 1 < n) ? byte
+                                                         : static_cast<uint8_t>((codes[i0 / 2 + b] & 0xF0u) | (byte & 0x0Fu));
+            }
+        }
+        if (any && (u & 3u) == 0u) scale[u >> 2] = m;
+    }
+}
+
+std::atomic<int> g_q4_grid[64];
+
+}  // namespace
+
+void q4_levels_host(float out[16]) {
+    for (int i = 0; i < 16; ++i) out[i] = kQ4Level[i];
+}
+
+cudaError_t launch_q4_perturb(const Q4Params& p, int grid_ctas, cudaStream_t stream) {
+    if (p.n_units == 0) return cudaSuccess;
+    int grid = grid_ctas;
+    if (grid <= 0) {
+        int dev = 0;
+        cudaError_t err = cudaGetDevice(&dev);
+        if (err != cudaSuccess) return err;
+        grid = dev < 64 ? g_q4_grid[dev].load(std::memory_order_relaxed) : 0;
+        if (grid <= 0) {
+            int sms = 0, per_sm = 0;
+            err = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+            if (err != cudaSuccess) return err;
+            err = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, q4_perturb_kernel,
+                                                                kThreadsQ4, 0);
+            if (err != cudaSuccess) return err;
+            grid = sms * (per_sm > 0 ? per_sm : 1);
+            if (dev < 64) g_q4_grid[dev].store(grid, std::memory_order_relaxed);
+        }
+        const uint64_t needed = (p.n_units + kThreadsQ4 - 1) / kThreadsQ4;
+        if (needed < static_cast<uint64_t>(grid)) grid = static_cast<int>(needed);
+    }
+    q4_perturb_kernel<<<grid, kThreadsQ4, 0, stream>>>(p);
+    return cudaGetLastError();
+}
+
+}  // namespace jb

@@ -202,3 +202,20 @@ def test_checksum_validation(jb):
     assert L.jb_checksum(src, 1, 0, None, None) == -1
     assert L.jb_checksum(src, 1, 0, C.c_void_p(FAKE + 4), None) == -3
     assert L.jb_checksum(src, 1, 3, C.c_void_p(FAKE), None) == -2
+
+
+def test_q4_levels_match_oracle_and_validation(jb):
+    import ctypes as C
+    assert np.array_equal(jb.jb_q4_levels(), oracle.q4_levels())
+    L = jb.lib()
+    seg = (jb.jb_q4_segment * 1)()
+    seg[0] = jb.jb_q4_segment(FAKE, FAKE + 4096, 100, 8)
+    assert L.jb_perturb_q4(seg, 1, jb.jb_seed(1, 0, 0), float("nan"), None) == -1
+    seg[0] = jb.jb_q4_segment(FAKE + 4, FAKE + 4096, 100, 8)       # codes not 8-byte aligned
+    assert L.jb_perturb_q4(seg, 1, jb.jb_seed(1, 0, 0), 1e-3, None) == -3
+    seg[0] = jb.jb_q4_segment(FAKE, FAKE + 4096, 100, 6)           # flat offset not a multiple of 4
+    assert L.jb_perturb_q4(seg, 1, jb.jb_seed(1, 0, 0), 1e-3, None) == -3
+    seg[0] = jb.jb_q4_segment(FAKE, FAKE + 40, 100, 8)             # scales overlap the codes
+    assert L.jb_perturb_q4(seg, 1, jb.jb_seed(1, 0, 0), 1e-3, None) == -1
+    seg[0] = jb.jb_q4_segment(0, FAKE, 100, 8)
+    assert L.jb_perturb_q4(seg, 1, jb.jb_seed(1, 0, 0), 1e-3, None) == -1
