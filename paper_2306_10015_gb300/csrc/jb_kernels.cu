@@ -163,6 +163,69 @@ struct Tile {
     bool full[V];
 };
 
+__device__ __forceinline__ uint64_t dst_address(const SegParam& g) { return g.ptr & ~1ull; }
+__device__ __forceinline__ uint64_t dst_address(const SegParamOut& g) { return g.dst; }
+
+// Warp-uniform description of a warp tile that lies inside one segment with every
+// vector full and on the 16-byte path (the common case): vector 32 j + lane of the
+// tile is at base + (32 j + lane) * 16 bytes and starts at global window
+// win0 + 32 j + lane. Every lane computes the same values, so branching on `fast`
+// does not diverge; other tiles take the per-vector path of load_tile/store_tile.
+struct TileFast {
+    bool fast;
+    uint32_t count;  // vectors in the tile
+    uint64_t base;   // source address of the tile's first vector
+    uint64_t dst;    // destination address of the tile's first vector
+    uint64_t win0;   // global window (E-element group) of the first vector
+};
+
+template <int E, int V, int ES, typename P>
+__device__ __forceinline__ TileFast tile_fast(const P& p, uint64_t wt, uint32_t& s) {
+    const uint64_t v0 = wt * (32u * V);
+    const uint64_t n_vec = p.n_vec;
+    while (s + 1 < p.n_segs && p.segs[s + 1].vec0 <= v0) ++s;
+    const auto& g = p.segs[s];
+    const uint64_t seg_end = s + 1 < p.n_segs ? p.segs[s + 1].vec0 : n_vec;
+    const uint64_t vend = v0 + 32u * V < n_vec ? v0 + 32u * V : n_vec;
+    TileFast f;
+    f.win0 = g.fo / E + (v0 - g.vec0);
+    const int64_t i_first = static_cast<int64_t>(f.win0 * E) - static_cast<int64_t>(g.fo);
+    const int64_t i_end = i_first + static_cast<int64_t>(vend - v0) * E;
+    f.fast = vend <= seg_end && (g.ptr & 1ull) && i_first >= 0 && i_end <= static_cast<int64_t>(g.n);
+    f.count = static_cast<uint32_t>(vend - v0);
+    f.base = (g.ptr & ~1ull) + static_cast<uint64_t>(i_first) * ES;
+    f.dst = dst_address(g) + static_cast<uint64_t>(i_first) * ES;
+    return f;
+}
+
+template <typename T, int V>
+__device__ __forceinline__ void load_tile_fast(const TileFast& f, uint32_t lane, Tile<T, V>& tl) {
+    constexpr int E = Traits<T>::E;
+#pragma unroll
+    for (int j = 0; j < V; ++j) {
+        const uint32_t v = 32u * j + lane;
+        tl.blk[j] = (f.win0 + v) * (E / 4);
+        tl.full[j] = v < f.count;
+        tl.seg[j] = 0;
+        if (tl.full[j]) {
+            load_vec(reinterpret_cast<const T*>(f.base + 16ull * v), tl.x[j]);
+        } else {
+#pragma unroll
+            for (int t = 0; t < E; ++t) tl.x[j][t] = 0.0f;
+        }
+    }
+}
+
+template <typename T, int V, bool TO_DST = false>
+__device__ __forceinline__ void store_tile_fast(const TileFast& f, uint32_t lane, const Tile<T, V>& tl) {
+#pragma unroll
+    for (int j = 0; j < V; ++j) {
+        const uint32_t v = 32u * j + lane;
+        if (v < f.count)
+            store_vec(reinterpret_cast<T*>((TO_DST ? f.dst : f.base) + 16ull * v), tl.x[j]);
+    }
+}
+
 // Loads tile wt. The segment cursor s only moves forward: a thread's vector
 // indices grow from one call to the next.
 template <typename T, int V, typename P>
@@ -330,10 +393,13 @@ __launch_bounds__(kThreads)
 
     for (uint64_t wt = warp; wt * (32u * V) < n_vec; wt += n_warps) {
         Tile<T, V> tl;
-        load_tile<T, V>(p, wt, lane, s, tl);
+        const TileFast f = tile_fast<Traits<T>::E, V, sizeof(T)>(p, wt, s);
+        if (f.fast) load_tile_fast<T, V>(f, lane, tl);
+        else load_tile<T, V>(p, wt, lane, s, tl);
         if constexpr (UPDATE) update_tile<T, V>(p, tl);
         else perturb_tile<T, V>(p, tl);
-        store_tile<T, V>(p, wt, lane, tl);
+        if (f.fast) store_tile_fast<T, V>(f, lane, tl);
+        else store_tile<T, V>(p, wt, lane, tl);
     }
 }
 
@@ -349,7 +415,9 @@ __global__ void __launch_bounds__(kThreads) general_update_kernel(const __grid_c
     uint32_t s = 0;
     for (uint64_t wt = warp; wt * (32u * V) < p.n_vec; wt += n_warps) {
         Tile<T, V> tl;
-        load_tile<T, V>(p, wt, lane, s, tl);
+        const TileFast f = tile_fast<Traits<T>::E, V, sizeof(T)>(p, wt, s);
+        if (f.fast) load_tile_fast<T, V>(f, lane, tl);
+        else load_tile<T, V>(p, wt, lane, s, tl);
         uint32_t kb = 0;
         for (uint32_t g = 0; g < p.n_groups; ++g) {
             const uint32_t ke = p.group_end[g];  // > kb: the host drops empty groups
@@ -358,8 +426,13 @@ __global__ void __launch_bounds__(kThreads) general_update_kernel(const __grid_c
             add_acc<T, V, true>(tl, acc);
             kb = ke;
         }
-        store_tile<T, V, true>(p, wt, lane, tl);
-        if (p.write_src) store_tile<T, V, false>(p, wt, lane, tl);
+        if (f.fast) {
+            store_tile_fast<T, V, true>(f, lane, tl);
+            if (p.write_src) store_tile_fast<T, V, false>(f, lane, tl);
+        } else {
+            store_tile<T, V, true>(p, wt, lane, tl);
+            if (p.write_src) store_tile<T, V, false>(p, wt, lane, tl);
+        }
     }
 }
 
@@ -413,6 +486,21 @@ __global__ void __launch_bounds__(kThreads) checksum_kernel(const __grid_constan
         uint4 w[V];
         uint64_t win[V];
         bool valid[V];
+        const TileFast f = tile_fast<E, V, sizeof(T)>(p, wt, s);
+        if (f.fast) {
+#pragma unroll
+            for (int j = 0; j < V; ++j) {
+                const uint32_t v = 32u * j + lane;
+                valid[j] = v < f.count;
+                win[j] = f.win0 + v;
+                w[j] = valid[j] ? __ldcs(reinterpret_cast<const uint4*>(f.base + 16ull * v))
+                                : make_uint4(0u, 0u, 0u, 0u);
+            }
+#pragma unroll
+            for (int j = 0; j < V; ++j)
+                if (valid[j]) sum += window_hash(win[j], w[j]);
+            continue;
+        }
 #pragma unroll
         for (int j = 0; j < V; ++j) {
             const uint64_t vi = wt * (32u * V) + 32u * j + lane;
