@@ -66,6 +66,19 @@ def parse():
     return ap.parse_args()
 
 
+def aggregate_ranks(ms_local: float, units_local: float, dist=None, device=None):
+    """Whole-job figures over ranks that ran independent replicas: the slowest
+    rank's time and the sum of the units all ranks processed."""
+    if dist is None or not dist.is_initialized() or dist.get_world_size() == 1:
+        return ms_local, units_local
+    import torch
+    t = torch.tensor([ms_local, units_local], dtype=torch.float64, device=device)
+    mx = t.clone()
+    dist.all_reduce(mx, op=dist.ReduceOp.MAX)
+    dist.all_reduce(t, op=dist.ReduceOp.SUM)
+    return float(mx[0].item()), float(t[1].item())
+
+
 def dist_env():
     return (int(os.environ.get("RANK", 0)), int(os.environ.get("LOCAL_RANK", 0)),
             int(os.environ.get("WORLD_SIZE", 1)))
@@ -271,12 +284,10 @@ def main():
     ms = e0.elapsed_time(e1)
     upd_ms = [x.elapsed_time(y) for x, y in zip(ev["u0"], ev["u1"])]
     pert_ms = [x.elapsed_time(y) / 3 for x, y in zip(ev["p0"], ev["u0"])]
-    if dist is not None:
-        tt = torch.tensor([ms], device="cuda")
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        ms = float(tt.item())
+    ms, units = aggregate_ranks(ms, float(N * (K + 3) * a.steps), dist,
+                                torch.device("cuda", local_rank))
     ms_per_step = ms / a.steps
-    units_per_step = N * (K + 3) * world
+    units_per_step = units / a.steps
     value = units_per_step / (ms_per_step / 1e3)
 
     # end to end through the same public calls, theta in pinned host memory: the
@@ -416,10 +427,7 @@ def run_e2e(a, jb, tensors, offs, seeds, codes, ghat, mids, own, stream, N, esiz
     z1.record(stream)
     torch.cuda.synchronize()
     h2d_ms, d2h_ms = y0.elapsed_time(y1), y1.elapsed_time(z1)
-    if dist is not None:
-        tt = torch.tensor([xms], device="cuda")
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        xms = float(tt.item())
+    xms, _ = aggregate_ranks(xms, 0.0, dist, torch.device("cuda", torch.cuda.current_device()))
     del host
     return {"value": units_per_step / (xms / 1e3), "unit": UNIT,
             "h2d_bytes_per_step": N * esize, "d2h_bytes_per_step": N * esize,
