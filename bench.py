@@ -506,29 +506,29 @@ def next_legs(a, jb, table, stream):
     import synthetic
     out = []
     ev = lambda: torch.cuda.Event(enable_timing=True)
-    K = a.K
-    seeds = jb.seeds_array([(int(m), 9, 0) for m in synthetic.machine_ids(K, 920)])
-    q = synthetic.byte_codes(K, 920)
     backup = jb.ParamTable([torch.empty_like(t) for t in table.tensors], table.flat_offsets)
     for b, t in zip(backup.tensors, table.tensors):
         b.copy_(t)
-    for mode in ("copy+update", "fused", "fused+refresh"):
-        def once():
-            if mode == "copy+update":
-                for b, t in zip(backup.tensors, table.tensors):
-                    t.copy_(b)
-                jb.jb_apply_updates(table, seeds, q, a.lr, 1.0, a.qscale, stream)
-            else:
-                jb.jb_apply_updates_from(backup, table, seeds, q, a.lr, 1.0, a.qscale,
-                                         write_src=(mode == "fused+refresh"), stream=stream)
-        once()
-        x0, x1 = ev(), ev()
-        x0.record(stream)
-        for _ in range(2):
+    for K in sorted({1, 4, a.K}):
+        seeds = jb.seeds_array([(int(m), 9, 0) for m in synthetic.machine_ids(K, 920)])
+        q = synthetic.byte_codes(K, 920)
+        for mode in ("copy+update", "fused", "fused+refresh"):
+            def once():
+                if mode == "copy+update":
+                    for b, t in zip(backup.tensors, table.tensors):
+                        t.copy_(b)
+                    jb.jb_apply_updates(table, seeds, q, a.lr, 1.0, a.qscale, stream)
+                else:
+                    jb.jb_apply_updates_from(backup, table, seeds, q, a.lr, 1.0, a.qscale,
+                                             write_src=(mode == "fused+refresh"), stream=stream)
             once()
-        x1.record(stream)
-        torch.cuda.synchronize()
-        out.append({"leg": "restore+update", "mode": mode, "K": K, "ms": x0.elapsed_time(x1) / 2})
+            x0, x1 = ev(), ev()
+            x0.record(stream)
+            for _ in range(2):
+                once()
+            x1.record(stream)
+            torch.cuda.synchronize()
+            out.append({"leg": "restore+update", "mode": mode, "K": K, "ms": x0.elapsed_time(x1) / 2})
     del backup
     for T, Kt in ((16, 4), (64, 1)):
         steps = []

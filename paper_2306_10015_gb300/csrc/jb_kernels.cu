@@ -17,11 +17,12 @@
 // work: the cost is one HBM read and write of theta (2 sizeof(T) bytes per
 // element) against K Gaussians per element (a quarter Philox4x32-10 block and
 // half a Box-Muller transform each). The grid is persistent (a multiple of the
-// SM count times the resident CTAs per SM) and strides over warp tiles: a warp
-// tile is 32 * V consecutive 16-byte vectors, lane l taking vectors l, l + 32,
-// ..., so every load and store instruction of a warp covers 512 contiguous
-// bytes (fully coalesced, 128-bit per thread). Each thread keeps V vectors
-// (16 elements, 4 Philox blocks) in flight for instruction-level parallelism.
+// SM count times the resident CTAs per SM) and strides over spans of S warp
+// tiles: a warp tile is 32 * V consecutive 16-byte vectors, lane l taking
+// vectors l, l + 32, ..., so every load and store instruction of a warp covers
+// 512 contiguous bytes (fully coalesced, 128-bit per thread). Each thread keeps
+// V vectors in flight for instruction-level parallelism; the segment lookup
+// (64-bit index arithmetic) is paid once per span, not once per tile.
 // The K (seed, coefficient) pairs live in the kernel parameter space and are
 // read with warp-uniform indices (constant-bank broadcast). Accumulation is a
 // fixed-order fp32 FMA chain with no atomics: results are bitwise repeatable
@@ -54,7 +55,25 @@ namespace {
 #define JB_VP_F32 4
 #endif
 #ifndef JB_VP_BF16
-#define JB_VP_BF16 2
+#define JB_VP_BF16 4
+#endif
+#ifndef JB_SU_F32  // warp tiles per span, update kernels
+#define JB_SU_F32 4
+#endif
+#ifndef JB_SU_BF16
+#define JB_SU_BF16 4
+#endif
+#ifndef JB_SG_F32  // warp tiles per span, general update kernel
+#define JB_SG_F32 1
+#endif
+#ifndef JB_SG_BF16
+#define JB_SG_BF16 1
+#endif
+#ifndef JB_SP_F32  // warp tiles per span, perturb kernel
+#define JB_SP_F32 4
+#endif
+#ifndef JB_SP_BF16
+#define JB_SP_BF16 4
 #endif
 #ifndef JB_PIPE_F32
 #define JB_PIPE_F32 0
@@ -64,8 +83,9 @@ namespace {
 #endif
 
 // Per storage type: elements per 16-byte vector, vectors per thread per warp tile,
-// and whether the update loop computes seed k + 1's Philox words while seed k is
-// transformed (measured faster for bf16, slower for fp32 at these tile sizes).
+// warp tiles per span (the unit whose segment lookup is done once), and whether
+// the update loop computes seed k + 1's Philox words while seed k is transformed
+// (measured faster for bf16, slower for fp32 at these tile sizes).
 template <typename T>
 struct Traits;
 template <>
@@ -74,6 +94,9 @@ struct Traits<float> {
     static constexpr int V = JB_V_F32;
     static constexpr bool PIPE = JB_PIPE_F32;
     static constexpr int VP = JB_VP_F32;  // vectors per thread, perturb
+    static constexpr int SU = JB_SU_F32;  // tiles per span, update
+    static constexpr int SG = JB_SG_F32;  // tiles per span, general update
+    static constexpr int SP = JB_SP_F32;  // tiles per span, perturb
 };
 template <>
 struct Traits<__nv_bfloat16> {
@@ -81,6 +104,9 @@ struct Traits<__nv_bfloat16> {
     static constexpr int V = JB_V_BF16;
     static constexpr bool PIPE = JB_PIPE_BF16;
     static constexpr int VP = JB_VP_BF16;
+    static constexpr int SU = JB_SU_BF16;
+    static constexpr int SG = JB_SG_BF16;
+    static constexpr int SP = JB_SP_BF16;
 };
 
 __device__ __forceinline__ void load_vec(const float* p, float (&x)[4]) {
@@ -286,6 +312,54 @@ __device__ __forceinline__ void store_tile(const P& p, uint64_t wt, uint32_t lan
     }
 }
 
+// Runs op on each of this warp's tiles and stores the result (to the destination
+// table when TO_DST, and then also back to the source when also_src). The warp
+// takes spans of S consecutive warp tiles, strided by the number of warps in the
+// grid. The segment lookup and fast-path test are done once per span: when the
+// whole span lies inside one aligned segment, its tiles follow one another at
+// fixed byte strides; otherwise each tile takes the per-vector path. Which warp
+// handles a tile never changes a result: every element's value depends only on
+// its own stored value, its global index and the seeds.
+template <typename T, int V, int S, bool TO_DST, typename P, typename Op>
+__device__ __forceinline__ void visit_tiles(const P& p, bool also_src, Op&& op) {
+    constexpr int E = Traits<T>::E;
+    constexpr uint32_t kTileVec = 32u * V;
+    const uint32_t lane = threadIdx.x & 31u;
+    const uint64_t warp = (static_cast<uint64_t>(blockIdx.x) * kThreads + threadIdx.x) >> 5;
+    const uint64_t n_warps = (static_cast<uint64_t>(gridDim.x) * kThreads) >> 5;
+    const uint64_t n_vec = p.n_vec;
+    uint32_t s = 0;  // segment cursor; only moves forward
+    for (uint64_t ws = warp; ws * (kTileVec * S) < n_vec; ws += n_warps) {
+        const TileFast fs = tile_fast<E, V * S, sizeof(T)>(p, ws, s);
+        if (fs.fast) {
+            TileFast f = fs;
+#pragma unroll 1
+            for (uint32_t done = 0; done < fs.count; done += kTileVec) {
+                f.count = fs.count - done < kTileVec ? fs.count - done : kTileVec;
+                Tile<T, V> tl;
+                load_tile_fast<T, V>(f, lane, tl);
+                op(tl);
+                store_tile_fast<T, V, TO_DST>(f, lane, tl);
+                if (TO_DST && also_src) store_tile_fast<T, V, false>(f, lane, tl);
+                f.base += 16ull * kTileVec;
+                f.dst += 16ull * kTileVec;
+                f.win0 += kTileVec;
+            }
+        } else {
+#pragma unroll 1
+            for (int u = 0; u < S; ++u) {
+                const uint64_t wt = ws * S + u;
+                if (wt * kTileVec >= n_vec) break;
+                Tile<T, V> tl;
+                load_tile<T, V>(p, wt, lane, s, tl);
+                op(tl);
+                store_tile<T, V, TO_DST>(p, wt, lane, tl);
+                if (TO_DST && also_src) store_tile<T, V, false>(p, wt, lane, tl);
+            }
+        }
+    }
+}
+
 // acc = sum_{k in [kb, ke)} c_k z_k for the tile, in fp32, in seed order (ke > kb).
 template <typename T, int V, typename P>
 __device__ __forceinline__ void accumulate_range(const P& p, const uint64_t (&blk)[V], uint32_t kb,
@@ -385,22 +459,11 @@ __launch_bounds__(kThreads)
 #endif
     seeded_kernel(const __grid_constant__ P p) {
     constexpr int V = UPDATE ? Traits<T>::V : Traits<T>::VP;
-    const uint32_t lane = threadIdx.x & 31u;
-    const uint64_t warp = (static_cast<uint64_t>(blockIdx.x) * kThreads + threadIdx.x) >> 5;
-    const uint64_t n_warps = (static_cast<uint64_t>(gridDim.x) * kThreads) >> 5;
-    const uint64_t n_vec = p.n_vec;
-    uint32_t s = 0;  // segment cursor
-
-    for (uint64_t wt = warp; wt * (32u * V) < n_vec; wt += n_warps) {
-        Tile<T, V> tl;
-        const TileFast f = tile_fast<Traits<T>::E, V, sizeof(T)>(p, wt, s);
-        if (f.fast) load_tile_fast<T, V>(f, lane, tl);
-        else load_tile<T, V>(p, wt, lane, s, tl);
+    constexpr int S = UPDATE ? Traits<T>::SU : Traits<T>::SP;
+    visit_tiles<T, V, S, false>(p, false, [&](Tile<T, V>& tl) {
         if constexpr (UPDATE) update_tile<T, V>(p, tl);
         else perturb_tile<T, V>(p, tl);
-        if (f.fast) store_tile_fast<T, V>(f, lane, tl);
-        else store_tile<T, V>(p, wt, lane, tl);
-    }
+    });
 }
 
 // The generalised update: source -> destination (optionally also back to the
@@ -409,15 +472,7 @@ __launch_bounds__(kThreads)
 template <typename T>
 __global__ void __launch_bounds__(kThreads) general_update_kernel(const __grid_constant__ GeneralParams p) {
     constexpr int V = Traits<T>::V;
-    const uint32_t lane = threadIdx.x & 31u;
-    const uint64_t warp = (static_cast<uint64_t>(blockIdx.x) * kThreads + threadIdx.x) >> 5;
-    const uint64_t n_warps = (static_cast<uint64_t>(gridDim.x) * kThreads) >> 5;
-    uint32_t s = 0;
-    for (uint64_t wt = warp; wt * (32u * V) < p.n_vec; wt += n_warps) {
-        Tile<T, V> tl;
-        const TileFast f = tile_fast<Traits<T>::E, V, sizeof(T)>(p, wt, s);
-        if (f.fast) load_tile_fast<T, V>(f, lane, tl);
-        else load_tile<T, V>(p, wt, lane, s, tl);
+    visit_tiles<T, V, Traits<T>::SG, true>(p, p.write_src != 0, [&](Tile<T, V>& tl) {
         uint32_t kb = 0;
         for (uint32_t g = 0; g < p.n_groups; ++g) {
             const uint32_t ke = p.group_end[g];  // > kb: the host drops empty groups
@@ -426,14 +481,7 @@ __global__ void __launch_bounds__(kThreads) general_update_kernel(const __grid_c
             add_acc<T, V, true>(tl, acc);
             kb = ke;
         }
-        if (f.fast) {
-            store_tile_fast<T, V, true>(f, lane, tl);
-            if (p.write_src) store_tile_fast<T, V, false>(f, lane, tl);
-        } else {
-            store_tile<T, V, true>(p, wt, lane, tl);
-            if (p.write_src) store_tile<T, V, false>(p, wt, lane, tl);
-        }
-    }
+    });
 }
 
 // Model checksum (ChecksumMatch, Algorithm 1): the sum mod 2^64, over 16-byte
@@ -445,9 +493,13 @@ __global__ void __launch_bounds__(kThreads) general_update_kernel(const __grid_c
 constexpr uint32_t kSumKey0 = 0x6A09E667u, kSumKey1 = 0xF3BCC908u;
 constexpr int kSumRounds = 4;
 #ifndef JB_SUM_V
-#define JB_SUM_V 4
+#define JB_SUM_V 8
 #endif
 constexpr int kSumV = JB_SUM_V;  // 16-byte loads in flight per thread
+#ifndef JB_SUM_S
+#define JB_SUM_S 4
+#endif
+constexpr int kSumS = JB_SUM_S;  // warp tiles per span
 
 __device__ __forceinline__ uint64_t window_hash(uint64_t win, uint4 w) {
     uint32_t x0 = w.x, x1 = w.y, x2 = w.z, x3 = w.w;
@@ -469,65 +521,88 @@ __device__ __forceinline__ uint32_t raw_bits(const __nv_bfloat16* p) {
     return *reinterpret_cast<const uint16_t*>(p);
 }
 
+// Checksum terms of warp tile wt on the per-vector path (tiles that cross a
+// segment boundary or lie in a segment off the 16-byte grid): windows are read
+// element by element where they are partial, with elements outside the segment
+// taken as zero bits.
+template <typename T, int V>
+__device__ __forceinline__ uint64_t sum_tile_general(const PerturbParams& p, uint64_t wt, uint32_t lane,
+                                                     uint32_t& s) {
+    constexpr int E = Traits<T>::E;
+    constexpr int BITS = 8 * static_cast<int>(sizeof(T));
+    const uint64_t n_vec = p.n_vec;
+    const uint32_t n_segs = p.n_segs;
+    uint64_t sum = 0;
+#pragma unroll
+    for (int j = 0; j < V; ++j) {
+        const uint64_t vi = wt * (32u * V) + 32u * j + lane;
+        const bool valid = vi < n_vec;
+        if (valid)
+            while (s + 1 < n_segs && p.segs[s + 1].vec0 <= vi) ++s;
+        const SegParam& g = p.segs[s];
+        const uint64_t win = g.fo / E + (vi - g.vec0);
+        const int64_t i0 = static_cast<int64_t>(win * E) - static_cast<int64_t>(g.fo);
+        const int64_t n = static_cast<int64_t>(g.n);
+        const T* base = reinterpret_cast<const T*>(g.ptr & ~1ull);
+        uint4 w;
+        if (valid && (g.ptr & 1ull) && i0 >= 0 && i0 + E <= n) {
+            w = __ldcs(reinterpret_cast<const uint4*>(base + i0));
+        } else {
+            uint32_t ww[4] = {0u, 0u, 0u, 0u};
+#pragma unroll
+            for (int t = 0; t < E; ++t) {
+                const int64_t i = i0 + t;
+                if (valid && i >= 0 && i < n) ww[t * BITS / 32] |= raw_bits(base + i) << ((t * BITS) % 32);
+            }
+            w = make_uint4(ww[0], ww[1], ww[2], ww[3]);
+        }
+        if (valid) sum += window_hash(win, w);
+    }
+    return sum;
+}
+
 template <typename T>
 __global__ void __launch_bounds__(kThreads) checksum_kernel(const __grid_constant__ PerturbParams p,
                                                            unsigned long long* out) {
     constexpr int E = Traits<T>::E;
     constexpr int V = kSumV;
-    constexpr int BITS = 8 * static_cast<int>(sizeof(T));
     const uint32_t lane = threadIdx.x & 31u;
     const uint64_t warp = (static_cast<uint64_t>(blockIdx.x) * kThreads + threadIdx.x) >> 5;
     const uint64_t n_warps = (static_cast<uint64_t>(gridDim.x) * kThreads) >> 5;
     const uint64_t n_vec = p.n_vec;
-    const uint32_t n_segs = p.n_segs;
+    constexpr int S = kSumS;
+    constexpr uint32_t kTileVec = 32u * V;
     uint32_t s = 0;
     uint64_t sum = 0;
-    for (uint64_t wt = warp; wt * (32u * V) < n_vec; wt += n_warps) {
-        uint4 w[V];
-        uint64_t win[V];
-        bool valid[V];
-        const TileFast f = tile_fast<E, V, sizeof(T)>(p, wt, s);
-        if (f.fast) {
+    for (uint64_t ws = warp; ws * (kTileVec * S) < n_vec; ws += n_warps) {
+        const TileFast fs = tile_fast<E, V * S, sizeof(T)>(p, ws, s);
+        if (fs.fast) {
+#pragma unroll 1
+            for (uint32_t done = 0; done < fs.count; done += kTileVec) {
+                const uint64_t base = fs.base + 16ull * done;
+                uint4 w[V];
+                uint64_t win[V];
+                bool valid[V];
 #pragma unroll
-            for (int j = 0; j < V; ++j) {
-                const uint32_t v = 32u * j + lane;
-                valid[j] = v < f.count;
-                win[j] = f.win0 + v;
-                w[j] = valid[j] ? __ldcs(reinterpret_cast<const uint4*>(f.base + 16ull * v))
-                                : make_uint4(0u, 0u, 0u, 0u);
+                for (int j = 0; j < V; ++j) {
+                    const uint32_t v = 32u * j + lane;
+                    valid[j] = done + v < fs.count;
+                    win[j] = fs.win0 + done + v;
+                    w[j] = valid[j] ? __ldcs(reinterpret_cast<const uint4*>(base + 16ull * v))
+                                    : make_uint4(0u, 0u, 0u, 0u);
+                }
+#pragma unroll
+                for (int j = 0; j < V; ++j)
+                    if (valid[j]) sum += window_hash(win[j], w[j]);
             }
-#pragma unroll
-            for (int j = 0; j < V; ++j)
-                if (valid[j]) sum += window_hash(win[j], w[j]);
             continue;
         }
-#pragma unroll
-        for (int j = 0; j < V; ++j) {
-            const uint64_t vi = wt * (32u * V) + 32u * j + lane;
-            valid[j] = vi < n_vec;
-            if (valid[j])
-                while (s + 1 < n_segs && p.segs[s + 1].vec0 <= vi) ++s;
-            const SegParam& g = p.segs[s];
-            win[j] = g.fo / E + (vi - g.vec0);
-            const int64_t i0 = static_cast<int64_t>(win[j] * E) - static_cast<int64_t>(g.fo);
-            const int64_t n = static_cast<int64_t>(g.n);
-            const T* base = reinterpret_cast<const T*>(g.ptr & ~1ull);
-            if (valid[j] && (g.ptr & 1ull) && i0 >= 0 && i0 + E <= n) {
-                w[j] = __ldcs(reinterpret_cast<const uint4*>(base + i0));
-            } else {
-                uint32_t ww[4] = {0u, 0u, 0u, 0u};
-#pragma unroll
-                for (int t = 0; t < E; ++t) {
-                    const int64_t i = i0 + t;
-                    if (valid[j] && i >= 0 && i < n)
-                        ww[t * BITS / 32] |= raw_bits(base + i) << ((t * BITS) % 32);
-                }
-                w[j] = make_uint4(ww[0], ww[1], ww[2], ww[3]);
-            }
+#pragma unroll 1
+        for (int u = 0; u < S; ++u) {
+            const uint64_t wt = ws * S + u;
+            if (wt * kTileVec >= n_vec) break;
+            sum += sum_tile_general<T, V>(p, wt, lane, s);
         }
-#pragma unroll
-        for (int j = 0; j < V; ++j)
-            if (valid[j]) sum += window_hash(win[j], w[j]);
     }
     // CTA reduction; every thread reaches the barrier
 #pragma unroll
@@ -614,7 +689,7 @@ cudaError_t launch_seeded(const P& p, int slot, int grid_ctas, cudaStream_t stre
         cudaError_t err = persistent_grid(kernel, slot, &grid);
         if (err != cudaSuccess) return err;
         constexpr uint64_t vec_per_cta =
-            32ull * (UPDATE ? Traits<T>::V : Traits<T>::VP) * (kThreads / 32);
+            32ull * (UPDATE ? Traits<T>::V * Traits<T>::SU : Traits<T>::VP * Traits<T>::SP) * (kThreads / 32);
         const uint64_t needed = (p.n_vec + vec_per_cta - 1) / vec_per_cta;
         if (needed < static_cast<uint64_t>(grid)) grid = static_cast<int>(needed);
     }
@@ -637,7 +712,7 @@ cudaError_t launch_general_t(const GeneralParams& p, int slot, int grid_ctas, cu
     if (grid <= 0) {
         cudaError_t err = persistent_grid(kernel, slot, &grid);
         if (err != cudaSuccess) return err;
-        constexpr uint64_t vec_per_cta = 32ull * Traits<T>::V * (kThreads / 32);
+        constexpr uint64_t vec_per_cta = 32ull * Traits<T>::V * Traits<T>::SG * (kThreads / 32);
         const uint64_t needed = (p.n_vec + vec_per_cta - 1) / vec_per_cta;
         if (needed < static_cast<uint64_t>(grid)) grid = static_cast<int>(needed);
     }
@@ -659,7 +734,7 @@ cudaError_t launch_checksum_t(const PerturbParams& p, unsigned long long* out, i
     if (grid <= 0) {
         cudaError_t err = persistent_grid(kernel, slot, &grid);
         if (err != cudaSuccess) return err;
-        constexpr uint64_t vec_per_cta = 32ull * kSumV * (kThreads / 32);
+        constexpr uint64_t vec_per_cta = 32ull * kSumV * kSumS * (kThreads / 32);
         const uint64_t needed = (p.n_vec + vec_per_cta - 1) / vec_per_cta;
         if (needed < static_cast<uint64_t>(grid)) grid = static_cast<int>(needed);
     }
