@@ -10,8 +10,14 @@
 // path (global index flat_offset + i), then per block scale' = max |w'| and
 // code' = nearest level of w' / scale'. Codes and scales are rewritten in place.
 // A 64-element block is four consecutive lanes (16 elements each): its maximum
-// is two butterfly shuffles. Levels and midpoints live in shared memory, read
-// with data-dependent indices (16 distinct words: no bank conflicts).
+// is two butterfly shuffles. Levels live in shared memory, read with
+// data-dependent indices (16 distinct words: no bank conflicts).
+//
+// Nearest level = the number of midpoints strictly below x. Consecutive
+// midpoints are more than 1/16 apart, so each bucket [j/16, (j+1)/16) of
+// [-1, 1) holds at most one; with b = floor(16 x) (exact in fp32), the code is
+// (midpoints below the bucket) + (x > the bucket's midpoint, if any): one
+// shared-memory read and one comparison instead of a 4-step binary search.
 #include <cuda_bf16.h>
 
 #include <atomic>
@@ -39,24 +45,36 @@ __constant__ float c_mid[15] = {
     -0x1.18df40p-3f, -0x1.72d976p-5f, 0x1.4421acp-5f,  0x1.e9d14cp-4f,  0x1.9e843cp-3f,
     0x1.2969c0p-2f,  0x1.8c97d4p-2f,  0x1.ff3a68p-2f,  0x1.47c276p-1f,  0x1.b8654cp-1f};
 
-// Nearest level of x: the number of midpoints strictly below x, by binary search.
-__device__ __forceinline__ uint32_t q4_code(float x, const float* mid) {
-    uint32_t c = 0;
-    if (x > mid[c + 7]) c += 8;
-    if (x > mid[c + 3]) c += 4;
-    if (x > mid[c + 1]) c += 2;
-    if (x > mid[c + 0]) c += 1;
-    return c;
+// Nearest level of x (ties to the lower): the number of midpoints strictly below
+// x. bucket[j] = (the midpoint in [(j - 16)/16, (j - 15)/16) or +inf, the
+// number of midpoints below (j - 16)/16 as integer bits). x below -1 or NaN
+// takes bucket 0 (code 0, as no midpoint is below it); x at or above 15/16
+// takes bucket 31.
+__device__ __forceinline__ uint32_t q4_code(float x, const float2* bucket) {
+    const float xc = fmaxf(x, -1.0f);                   // NaN -> -1
+    const int b = min(__float2int_rd(16.0f * xc), 15);  // in [-16, 15]
+    const float2 e = bucket[b + 16];
+    return __float_as_uint(e.y) + (x > e.x ? 1u : 0u);
 }
 
 constexpr int kThreadsQ4 = 256;
 
 __global__ void __launch_bounds__(kThreadsQ4) q4_perturb_kernel(const __grid_constant__ Q4Params p) {
     __shared__ float level[16];
-    __shared__ float mid[16];
-    if (threadIdx.x < 16) {
-        level[threadIdx.x] = c_level[threadIdx.x];
-        mid[threadIdx.x] = threadIdx.x < 15 ? c_mid[threadIdx.x] : 2.0f;
+    __shared__ float2 bucket[32];
+    if (threadIdx.x < 16) level[threadIdx.x] = c_level[threadIdx.x];
+    if (threadIdx.x < 32) {
+        const float lo = static_cast<float>(static_cast<int>(threadIdx.x) - 16) * 0.0625f;
+        const float hi = lo + 0.0625f;
+        uint32_t below = 0;
+        float m = __int_as_float(0x7F800000);  // +inf: no midpoint in the bucket
+#pragma unroll
+        for (int k = 0; k < 15; ++k) {
+            const float md = c_mid[k];
+            below += md < lo ? 1u : 0u;
+            if (md >= lo && md < hi) m = md;
+        }
+        bucket[threadIdx.x] = make_float2(m, __uint_as_float(below));
     }
     __syncthreads();  // every thread reaches this before any work
 
@@ -123,7 +141,7 @@ __global__ void __launch_bounds__(kThreadsQ4) q4_perturb_kernel(const __grid_con
         // quantize again
         uint32_t ow[2] = {0u, 0u};
 #pragma unroll
-        for (int k = 0; k < 16; ++k) ow[k / 8] |= q4_code(__fmul_rn(w[k], inv), mid) << (4 * (k % 8));
+        for (int k = 0; k < 16; ++k) ow[k / 8] |= q4_code(__fmul_rn(w[k], inv), bucket) << (4 * (k % 8));
         if (full) {
             *reinterpret_cast<uint2*>(codes + i0 / 2) = make_uint2(ow[0], ow[1]);
         } else if (any) {

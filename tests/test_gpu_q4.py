@@ -95,3 +95,80 @@ def test_q4_perturb_parity(jb, eps):
         if n % 2 == 1:  # the unused high nibble of an odd tail is left as it was
             assert dc.cpu().numpy()[n // 2] >> 4 == c[n // 2] >> 4
     print(f"eps={eps}: codes decided differently within tolerance of a midpoint: {near_total}")
+
+
+def _check_codes(gc, want, w, scale_blocks, eps, mids):
+    """Codes equal the oracle's except within fp32 error of a midpoint."""
+    scale = np.repeat(scale_blocks.astype(np.float64), 64)[: w.size]
+    x = np.where(scale > 0, w / np.where(scale > 0, scale, 1), 0.0)
+    tol = (2e-6 * eps + 4e-7 * scale) / np.where(scale > 0, scale, 1) + 4e-7
+    d = np.abs(x[:, None] - mids[None, :])
+    near = d.min(axis=1) <= tol
+    j = d.argmin(axis=1)
+    return (gc == want) | (near & ((gc == j) | (gc == j + 1)))
+
+
+def test_q4_perturb_zero_blocks(jb):
+    """All-zero blocks: with eps = 0 they stay zero (scale 0, every code the zero
+    level); with eps > 0 they take the noise alone."""
+    sizes = [64 * 5 + 7, 130]
+    offs = offsets(sizes)
+    host, dev = [], []
+    for i, n in enumerate(sizes):
+        w = synthetic.normal_values(n, 0.02, 90 + i).astype(np.float64)
+        w[64:192] = 0.0 if n > 192 else w[64:192]
+        w[:64] = 0.0
+        codes, scale = oracle.q4_quantize(w)
+        host.append((codes, scale, n))
+        pad = np.zeros(codes.size + 16, dtype=np.uint8)
+        pad[: codes.size] = codes
+        dev.append((torch.from_numpy(pad).cuda(), torch.from_numpy(scale.copy()).cuda(), n))
+    table = jb.Q4Table(dev, offs)
+    jb.jb_perturb_q4(table, (9, 9, 9), 0.0)
+    torch.cuda.synchronize()
+    zero_code = int(np.argmin(np.abs(oracle.q4_levels())))
+    for (c, s, n), (dc, ds, _) in zip(host, dev):
+        assert np.array_equal(dc.cpu().numpy()[: c.size], c)
+        assert ds.cpu().numpy()[0] == 0.0
+        assert np.all(codes_of(dc.cpu().numpy(), n)[:64] == zero_code)
+    eps = float(F32(1e-3))
+    seed = (77, 1, 2)
+    jb.jb_perturb_q4(table, seed, eps)
+    torch.cuda.synchronize()
+    lev = oracle.q4_levels().astype(np.float64)
+    mids = (lev[:-1] + lev[1:]) / 2
+    for (c, s, n), (dc, ds, _), fo in zip(host, dev, offs):
+        oc, os_, w = oracle.q4_perturb(c, s, n, fo, seed, eps)
+        gs = ds.cpu().numpy()
+        assert np.all(np.abs(gs.astype(np.float64) - os_) <= 2e-6 * os_ + 2e-6 * eps)
+        ok = _check_codes(codes_of(dc.cpu().numpy(), n), codes_of(oc, n), w, os_, eps, mids)
+        assert np.all(ok), (n, np.nonzero(~ok)[0][:5])
+
+
+def test_q4_perturb_large_sampled(jb):
+    """A multi-tensor set of 2^24+ elements with ragged sizes, checked on 3000
+    random 64-element blocks, each block recomputed by the oracle on its own
+    (a block depends only on its own codes, scale and global indices)."""
+    sizes = [(1 << 23) + 64 * 3, 5_000_003, 64 * 37 + 1, (1 << 22) - 17]
+    offs = offsets(sizes)
+    host, dev, table = make(jb, sizes, offs, stream=95)
+    seed = (0x1234_5678_9ABC, 3, 0)
+    eps = float(F32(1e-2))
+    jb.jb_perturb_q4(table, seed, eps)
+    torch.cuda.synchronize()
+    lev = oracle.q4_levels().astype(np.float64)
+    mids = (lev[:-1] + lev[1:]) / 2
+    rng = synthetic.rng(96)
+    n_bad = 0
+    for (c, s, n), (dc, ds, _), fo in zip(host, dev, offs):
+        gcodes, gscale = dc.cpu().numpy(), ds.cpu().numpy()
+        n_blocks = (n + 63) // 64
+        for b in rng.choice(n_blocks, size=min(n_blocks, 750), replace=False):
+            m = min(64, n - 64 * b)
+            cb = c[32 * b: 32 * b + (m + 1) // 2]
+            oc, os_, w = oracle.q4_perturb(cb, s[b: b + 1], m, fo + 64 * b, seed, eps)
+            assert abs(float(gscale[b]) - float(os_[0])) <= 2e-6 * float(os_[0]) + 2e-6 * eps, (n, b)
+            got = codes_of(gcodes[32 * b: 32 * b + (m + 1) // 2], m)
+            ok = _check_codes(got, codes_of(oc, m), w, os_, eps, mids)
+            n_bad += int(np.sum(~ok))
+    assert n_bad == 0
