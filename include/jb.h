@@ -79,7 +79,8 @@ typedef enum {
     JB_ERR_DUPLICATE_SEED = -4,   /* two pairs with the same (machine_id, step, sample_id) */
     JB_ERR_CUDA = -5,             /* a CUDA runtime call or launch failed */
     JB_ERR_RANGE = -6,            /* a coefficient -lr deq(q) / denom is not finite in fp32 */
-    JB_ERR_TOO_MANY_SEEDS = -7    /* K above jb_max_seeds_per_call() */
+    JB_ERR_TOO_MANY_SEEDS = -7,   /* K above jb_max_seeds_per_call() */
+    JB_ERR_NO_MEMORY = -8         /* host memory for the call's working copy could not be had */
 } jb_status;
 
 typedef enum { JB_F32 = 0, JB_BF16 = 1 } jb_dtype;
@@ -238,16 +239,19 @@ const char* jb_status_string(int status);
  * Test hooks (not on the hot path). Device buffers are caller-owned.
  * ------------------------------------------------------------------------- */
 
-/* d_out[4 i + w] = word w of Philox block first_block + i under `seed`. */
+/* d_out[4 i + w] = word w of Philox block first_block + i under `seed`.
+ * d_out must be 16-byte aligned (JB_ERR_MISALIGNED); n_blocks <= 2^38. */
 int jb_debug_philox(jb_seed seed, uint64_t first_block, uint64_t n_blocks, uint32_t* d_out,
                     struct CUstream_st* stream);
 
-/* d_out[i] = z of global element first_elem + i under `seed` (fp32). */
+/* d_out[i] = z of global element first_elem + i under `seed` (fp32).
+ * d_out must be 4-byte aligned (JB_ERR_MISALIGNED); n <= 2^38. */
 int jb_debug_gaussian(jb_seed seed, uint64_t first_elem, uint64_t n, float* d_out,
                       struct CUstream_st* stream);
 
 /* Box-Muller of raw word pairs: d_out[2 i], d_out[2 i + 1] = z of the even and
- * odd element for words (d_words[2 i], d_words[2 i + 1]). */
+ * odd element for words (d_words[2 i], d_words[2 i + 1]). Both buffers must be
+ * 4-byte aligned (JB_ERR_MISALIGNED); n_pairs <= 2^38. */
 int jb_debug_box_muller(const uint32_t* d_words, uint64_t n_pairs, float* d_out,
                         struct CUstream_st* stream);
 

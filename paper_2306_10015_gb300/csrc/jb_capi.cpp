@@ -9,6 +9,7 @@
 #include <algorithm>
 #include <cmath>
 #include <cstring>
+#include <new>
 #include <vector>
 
 #include "jb.h"
@@ -25,6 +26,22 @@ struct Seg {
 };
 
 size_t elem_size(int dtype) { return dtype == JB_F32 ? 4 : 2; }
+
+// [p, p + n * es) fits in the address space (written so that n * es cannot wrap).
+bool range_fits(uint64_t p, uint64_t n, uint64_t es) { return n <= (UINT64_MAX - p) / es; }
+
+// Runs an entry point's body; a host allocation failure (or any other C++
+// exception) becomes a status instead of crossing the C interface.
+template <typename F>
+int guarded(F&& body) noexcept {
+    try {
+        return body();
+    } catch (const std::bad_alloc&) {
+        return JB_ERR_NO_MEMORY;
+    } catch (...) {
+        return JB_ERR_INVALID_ARG;
+    }
+}
 int elems_per_vec(int dtype) { return dtype == JB_F32 ? 4 : 8; }
 
 // Checks the segment table; drops empty segments. Overlap in memory or in
@@ -42,7 +59,7 @@ int collect_segments(const jb_segment* segs, int n_segs, int dtype, std::vector<
         if (p == 0) return JB_ERR_INVALID_ARG;
         if (p % es != 0) return JB_ERR_MISALIGNED;
         if (s.numel > kMaxIndex || s.flat_offset > kMaxIndex - s.numel) return JB_ERR_INVALID_ARG;
-        if (p > UINT64_MAX - s.numel * es) return JB_ERR_INVALID_ARG;
+        if (!range_fits(p, s.numel, es)) return JB_ERR_INVALID_ARG;
         out.push_back({p, s.flat_offset, s.numel});
     }
     std::vector<Seg> by_fo(out), by_ptr(out);
@@ -187,7 +204,7 @@ int collect_destinations(const jb_segment* src, const jb_segment* dst, int n_seg
         const uint64_t p = reinterpret_cast<uint64_t>(dst[i].ptr);
         if (p == 0) return JB_ERR_INVALID_ARG;
         if (p % es != 0) return JB_ERR_MISALIGNED;
-        if (p > UINT64_MAX - dst[i].numel * es) return JB_ERR_INVALID_ARG;
+        if (!range_fits(p, dst[i].numel, es)) return JB_ERR_INVALID_ARG;
         dptr.push_back(p);
         const uint64_t sp = reinterpret_cast<uint64_t>(src[i].ptr);
         iv.push_back({sp, sp + src[i].numel * es, i, false});
@@ -321,39 +338,44 @@ JB_EXPORT int jb_apply_updates_from(const jb_segment* src, const jb_segment* dst
                                     struct CUstream_st* stream) {
     if (dst == nullptr && n_segs > 0) return JB_ERR_INVALID_ARG;
     if (K < 0) return JB_ERR_INVALID_ARG;
-    return general_impl(src, dst, n_segs, dtype, seeds, q, &K, 1, &lr, &denom, qscale, write_src,
-                        0, stream);
+    return guarded([&] {
+        return general_impl(src, dst, n_segs, dtype, seeds, q, &K, 1, &lr, &denom, qscale, write_src,
+                            0, stream);
+    });
 }
 
 JB_EXPORT int jb_replay_updates(const jb_segment* segs, int n_segs, int dtype, const jb_seed* seeds,
                                 const int8_t* q, const int* step_sizes, int n_steps,
                                 const float* lr, const float* denom, float qscale,
                                 struct CUstream_st* stream) {
-    return general_impl(segs, nullptr, n_segs, dtype, seeds, q, step_sizes, n_steps, lr, denom,
-                        qscale, 0, 0, stream);
+    return guarded([&] {
+        return general_impl(segs, nullptr, n_segs, dtype, seeds, q, step_sizes, n_steps, lr, denom,
+                            qscale, 0, 0, stream);
+    });
 }
 
 JB_EXPORT int jb_perturb(const jb_segment* segs, int n_segs, int dtype, jb_seed seed, float eps,
                          struct CUstream_st* stream) {
-    return perturb_impl(segs, n_segs, dtype, seed, eps, 0, stream);
+    return guarded([&] { return perturb_impl(segs, n_segs, dtype, seed, eps, 0, stream); });
 }
 
 JB_EXPORT int jb_perturb_with_grid(const jb_segment* segs, int n_segs, int dtype, jb_seed seed,
                                    float eps, int grid_ctas, struct CUstream_st* stream) {
-    return perturb_impl(segs, n_segs, dtype, seed, eps, grid_ctas, stream);
+    return guarded([&] { return perturb_impl(segs, n_segs, dtype, seed, eps, grid_ctas, stream); });
 }
 
 JB_EXPORT int jb_apply_updates(const jb_segment* segs, int n_segs, int dtype, const jb_seed* seeds,
                                const int8_t* q, int K, float lr, float denom, float qscale,
                                struct CUstream_st* stream) {
-    return update_impl(segs, n_segs, dtype, seeds, q, K, lr, denom, qscale, 0, stream);
+    return guarded([&] { return update_impl(segs, n_segs, dtype, seeds, q, K, lr, denom, qscale, 0, stream); });
 }
 
 JB_EXPORT int jb_apply_updates_with_grid(const jb_segment* segs, int n_segs, int dtype,
                                          const jb_seed* seeds, const int8_t* q, int K, float lr,
                                          float denom, float qscale, int grid_ctas,
                                          struct CUstream_st* stream) {
-    return update_impl(segs, n_segs, dtype, seeds, q, K, lr, denom, qscale, grid_ctas, stream);
+    return guarded(
+        [&] { return update_impl(segs, n_segs, dtype, seeds, q, K, lr, denom, qscale, grid_ctas, stream); });
 }
 
 namespace {
@@ -381,16 +403,16 @@ int checksum_impl(const jb_segment* segs, int n_segs, int dtype, uint64_t* d_out
 
 JB_EXPORT int jb_checksum(const jb_segment* segs, int n_segs, int dtype, uint64_t* d_out,
                           struct CUstream_st* stream) {
-    return checksum_impl(segs, n_segs, dtype, d_out, 0, stream);
+    return guarded([&] { return checksum_impl(segs, n_segs, dtype, d_out, 0, stream); });
 }
 
 JB_EXPORT int jb_checksum_with_grid(const jb_segment* segs, int n_segs, int dtype, uint64_t* d_out,
                                     int grid_ctas, struct CUstream_st* stream) {
-    return checksum_impl(segs, n_segs, dtype, d_out, grid_ctas, stream);
+    return guarded([&] { return checksum_impl(segs, n_segs, dtype, d_out, grid_ctas, stream); });
 }
 
-JB_EXPORT int jb_perturb_q4(const jb_q4_segment* segs, int n_segs, jb_seed seed, float eps,
-                            struct CUstream_st* stream) {
+namespace {
+int perturb_q4_impl(const jb_q4_segment* segs, int n_segs, jb_seed seed, float eps, cudaStream_t stream) {
     if (n_segs < 0 || (n_segs > 0 && segs == nullptr)) return JB_ERR_INVALID_ARG;
     if (!std::isfinite(eps)) return JB_ERR_INVALID_ARG;
     struct Q { uint64_t codes, scale, fo, n; };
@@ -439,6 +461,12 @@ JB_EXPORT int jb_perturb_q4(const jb_q4_segment* segs, int n_segs, jb_seed seed,
     }
     return JB_OK;
 }
+}  // namespace
+
+JB_EXPORT int jb_perturb_q4(const jb_q4_segment* segs, int n_segs, jb_seed seed, float eps,
+                            struct CUstream_st* stream) {
+    return guarded([&] { return perturb_q4_impl(segs, n_segs, seed, eps, stream); });
+}
 
 JB_EXPORT int jb_q4_levels(float* out) {
     if (out == nullptr) return JB_ERR_INVALID_ARG;
@@ -478,6 +506,7 @@ JB_EXPORT const char* jb_status_string(int status) {
         case JB_ERR_CUDA: return "CUDA runtime or launch error";
         case JB_ERR_RANGE: return "update coefficient not finite in fp32";
         case JB_ERR_TOO_MANY_SEEDS: return "more seeds than one call accepts";
+        case JB_ERR_NO_MEMORY: return "host memory allocation failed";
         default: return "unknown status";
     }
 }
@@ -495,6 +524,7 @@ JB_EXPORT int jb_debug_gaussian(jb_seed seed, uint64_t first_elem, uint64_t n, f
                                 struct CUstream_st* stream) {
     if (n > 0 && d_out == nullptr) return JB_ERR_INVALID_ARG;
     if (n > (1ull << 38) || first_elem > kMaxIndex - n) return JB_ERR_INVALID_ARG;
+    if (reinterpret_cast<uint64_t>(d_out) & 3ull) return JB_ERR_MISALIGNED;
     return cuda_status(jb::launch_debug_gaussian(seed_param(seed, 0.0f), first_elem, n, d_out, stream));
 }
 
@@ -502,5 +532,7 @@ JB_EXPORT int jb_debug_box_muller(const uint32_t* d_words, uint64_t n_pairs, flo
                                   struct CUstream_st* stream) {
     if (n_pairs > 0 && (d_words == nullptr || d_out == nullptr)) return JB_ERR_INVALID_ARG;
     if (n_pairs > (1ull << 38)) return JB_ERR_INVALID_ARG;
+    if ((reinterpret_cast<uint64_t>(d_words) | reinterpret_cast<uint64_t>(d_out)) & 3ull)
+        return JB_ERR_MISALIGNED;
     return cuda_status(jb::launch_debug_box_muller(d_words, n_pairs, d_out, stream));
 }

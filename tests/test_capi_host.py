@@ -47,7 +47,7 @@ def test_library_exports_every_declared_symbol(jb):
 
 
 def test_status_strings(jb):
-    for rc in range(-7, 1):
+    for rc in range(-8, 1):
         assert jb.jb_status_string(rc) not in ("", "unknown status")
     assert jb.jb_status_string(17) == "unknown status"
 
@@ -127,6 +127,10 @@ def test_invalid_arguments(jb):
     assert _perturb(jb, _segs(jb, [(FAKE, 10, 0), (FAKE + 4096, 10, 9)]), 2) == E["inv"]
     assert _perturb(jb, _segs(jb, [(FAKE, 10, 0), (FAKE + 36, 10, 100)]), 2) == E["inv"]
     assert _perturb(jb, _segs(jb, [(FAKE, 10, (1 << 62) - 5)]), 1) == E["inv"]
+    # a segment that would run past the end of the address space, including the
+    # case where numel * sizeof(T) itself is 2^64
+    assert _perturb(jb, _segs(jb, [(16, 1 << 62, 0)]), 1, dtype=0) == E["inv"]
+    assert _perturb(jb, _segs(jb, [((1 << 64) - 64, 100, 0)]), 1, dtype=1) == E["inv"]
     seeds = [(1, 0, 0), (2, 0, 0)]
     assert _update(jb, ok, 1, seeds + [(1, 0, 0)], [1, 2, 3]) == E["dup"]
     assert _update(jb, ok, 1, seeds, [1, 2], K=-1) == E["inv"]
@@ -219,3 +223,14 @@ def test_q4_levels_match_oracle_and_validation(jb):
     assert L.jb_perturb_q4(seg, 1, jb.jb_seed(1, 0, 0), 1e-3, None) == -1
     seg[0] = jb.jb_q4_segment(0, FAKE, 100, 8)
     assert L.jb_perturb_q4(seg, 1, jb.jb_seed(1, 0, 0), 1e-3, None) == -1
+
+
+def test_debug_hooks_check_alignment(jb):
+    """The test hooks refuse buffers their kernels could not store to or load from."""
+    L, seed = jb.lib(), jb.jb_seed(1, 2, 3)
+    assert L.jb_debug_philox(seed, 0, 4, ctypes.c_void_p(FAKE + 8), None) == -3
+    assert L.jb_debug_gaussian(seed, 0, 4, ctypes.c_void_p(FAKE + 2), None) == -3
+    assert L.jb_debug_box_muller(ctypes.c_void_p(FAKE + 1), 4, ctypes.c_void_p(FAKE), None) == -3
+    assert L.jb_debug_box_muller(ctypes.c_void_p(FAKE), 4, ctypes.c_void_p(FAKE + 2), None) == -3
+    assert L.jb_debug_gaussian(seed, 0, (1 << 38) + 1, ctypes.c_void_p(FAKE), None) == -1
+    assert L.jb_debug_gaussian(seed, 0, 4, None, None) == -1
