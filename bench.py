@@ -182,6 +182,15 @@ def oracle_rate(a, target_s: float):
     return n * (a.K + 3) / t, cores, t, n
 
 
+def bench_config(a, world):
+    """The workload description both arms print (sizes from the OPT shapes alone)."""
+    import synthetic
+    specs = synthetic.opt_tensors(a.model)
+    return {"workload": workload_name(a), "n_params": sum(sp.numel for sp in specs),
+            "n_tensors": len(specs), "K": a.K, "eps": a.eps, "lr": a.lr, "qscale": a.qscale,
+            "l2": "inputs larger than L2 (no flush needed)", "parallelism": f"replicas x{world}"}
+
+
 def run_reference(a):
     rank, _, world = dist_env()
     if rank != 0:
@@ -199,7 +208,7 @@ def run_reference(a):
         "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": a.gpus,
         "steps": a.steps, "warmup": a.warmup, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-        "config": {"workload": workload_name(a), "K": a.K},
+        "config": bench_config(a, world),
         "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
                          "sample": sample},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
@@ -339,10 +348,7 @@ def main():
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": a.steps,
         "warmup": a.warmup, "ms_per_step": ms_per_step, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": a.dtype, "data": "synthetic",
-        "config": {"workload": workload_name(a), "n_params": N, "n_tensors": table.n_segments,
-                   "K": K, "eps": a.eps, "lr": a.lr, "qscale": a.qscale,
-                   "l2": "inputs larger than L2 (no flush needed)",
-                   "parallelism": f"replicas x{world}"},
+        "config": bench_config(a, world),
         "hbm_gbs_step": step_bytes * world / (ms_per_step / 1e3) / 1e9,
         "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e,
         "gpu_launches": launches_per_step * a.steps, "clocks": clk,
@@ -451,15 +457,19 @@ def run_e2e(a, jb, tensors, offs, seeds, codes, ghat, mids, own, stream, N, esiz
             "ms_per_step": xms, "groups": len(groups), "h2d_ms": h2d_ms, "d2h_ms": d2h_ms}
 
 
+# The sources the update kernel's device code and launch shape are built from.
+UPDATE_KERNEL_SOURCES = ("jb_internal.h", "jb_kernels.cu", "jb_rng.cuh")
+
+
 def kernel_sources_digest() -> str:
-    """sha1 over the CUDA sources; ncu counters are valid only for the build they measured."""
+    """sha1 over the update kernel's sources; its ncu counters are valid only for
+    the build they measured."""
     import hashlib
     csrc = os.path.join(ROOT, "paper_2306_10015_gb300", "csrc")
     h = hashlib.sha1()
-    for name in sorted(os.listdir(csrc)):
-        if name.endswith((".cu", ".cuh", ".h", ".cpp")):
-            with open(os.path.join(csrc, name), "rb") as f:
-                h.update(name.encode() + b"\0" + f.read())
+    for name in UPDATE_KERNEL_SOURCES:
+        with open(os.path.join(csrc, name), "rb") as f:
+            h.update(name.encode() + b"\0" + f.read())
     return h.hexdigest()
 
 
