@@ -360,71 +360,89 @@ def main():
         dist.destroy_process_group()
 
 
-def run_e2e(a, jb, tensors, offs, seeds, codes, ghat, mids, own, stream, N, esize,
-            units_per_step, dist, n_groups=32):
-    """The step end to end with theta in pinned host memory.
+class E2EPipeline:
+    """Theta in pinned host memory, one step at a time through the public calls.
 
-    The 644 tensors are split into n_groups groups of consecutive tensors of about
+    The tensors are split into n_groups groups of consecutive tensors of about
     equal bytes. Each group lives in one pinned host buffer and one device buffer,
     and its tensors are views into them (64-element aligned), so a group moves in
     one copy each way. Three streams pipeline the groups: group g + 1 arrives while
     group g is transformed, and group g - 1 leaves. z depends only on the global
     index, so any split of the table gives the same bits."""
-    import torch
-    total = sum(t.numel() for t in tensors)
-    groups, cur, acc = [], [], 0
-    for i, t in enumerate(tensors):
-        cur.append(i)
-        acc += t.numel()
-        if acc >= total * (len(groups) + 1) / n_groups and len(groups) < n_groups - 1:
-            groups.append(cur)
-            cur = []
-    if cur:
-        groups.append(cur)
-    pad = lambda n: -(-n // 64) * 64
-    dev_bufs, host_bufs, views = [], [], [None] * len(tensors)
-    for g in groups:
-        n = sum(pad(tensors[i].numel()) for i in g)
-        d = torch.empty(n, dtype=tensors[0].dtype, device=tensors[0].device)
-        h = torch.empty(n, dtype=tensors[0].dtype, pin_memory=True)
-        o = 0
-        for i in g:
-            m = tensors[i].numel()
-            views[i] = d[o:o + m].view(tensors[i].shape)
-            views[i].copy_(tensors[i])
-            o += pad(m)
-        h.copy_(d)
-        dev_bufs.append(d)
-        host_bufs.append(h)
-    torch.cuda.synchronize()
-    copy_bytes = sum(b.numel() for b in dev_bufs) * esize
-    tables = [jb.ParamTable([views[i] for i in g], [offs[i] for i in g]) for g in groups]
-    s_in, s_out = torch.cuda.Stream(), torch.cuda.Stream()
-    out_done = [None] * len(groups)
 
-    def step(t):
-        s_own = (int(mids[own]), t, 0)
-        q = codes[t]
-        q[own] = jb.jb_quantize_grad(float(ghat[t]), a.qscale)
-        for gi, tab in enumerate(tables):
-            if out_done[gi] is not None:
-                s_in.wait_event(out_done[gi])
-            with torch.cuda.stream(s_in):
-                dev_bufs[gi].copy_(host_bufs[gi], non_blocking=True)
+    def __init__(self, jb, tensors, offs, stream, n_groups=32):
+        import torch
+        self.jb, self.stream = jb, stream
+        total = sum(t.numel() for t in tensors)
+        groups, cur, acc = [], [], 0
+        for i, t in enumerate(tensors):
+            cur.append(i)
+            acc += t.numel()
+            if acc >= total * (len(groups) + 1) / n_groups and len(groups) < n_groups - 1:
+                groups.append(cur)
+                cur = []
+        if cur:
+            groups.append(cur)
+        pad = lambda n: -(-n // 64) * 64
+        self.dev_bufs, self.host_bufs = [], []
+        self.views, self.host_views = [None] * len(tensors), [None] * len(tensors)
+        for g in groups:
+            n = sum(pad(tensors[i].numel()) for i in g)
+            d = torch.empty(n, dtype=tensors[0].dtype, device=tensors[0].device)
+            h = torch.empty(n, dtype=tensors[0].dtype, pin_memory=True)
+            o = 0
+            for i in g:
+                m = tensors[i].numel()
+                self.views[i] = d[o:o + m].view(tensors[i].shape)
+                self.views[i].copy_(tensors[i])
+                self.host_views[i] = h[o:o + m].view(tensors[i].shape)
+                o += pad(m)
+            h.copy_(d)
+            self.dev_bufs.append(d)
+            self.host_bufs.append(h)
+        torch.cuda.synchronize()
+        self.groups = groups
+        self.copy_bytes = sum(b.numel() * b.element_size() for b in self.dev_bufs)
+        self.tables = [jb.ParamTable([self.views[i] for i in g], [offs[i] for i in g]) for g in groups]
+        self.s_in, self.s_out = torch.cuda.Stream(), torch.cuda.Stream()
+        self.out_done = [None] * len(groups)
+
+    def step(self, s_own, seeds, q, eps, lr, qscale):
+        """Enqueue one step: per group copy in, perturb +eps/-2 eps/+eps, update, copy out."""
+        import torch
+        jb, stream = self.jb, self.stream
+        for gi, tab in enumerate(self.tables):
+            if self.out_done[gi] is not None:
+                self.s_in.wait_event(self.out_done[gi])
+            with torch.cuda.stream(self.s_in):
+                self.dev_bufs[gi].copy_(self.host_bufs[gi], non_blocking=True)
             arrived = torch.cuda.Event()
-            arrived.record(s_in)
+            arrived.record(self.s_in)
             stream.wait_event(arrived)
-            jb.jb_perturb(tab, s_own, a.eps, stream)
-            jb.jb_perturb(tab, s_own, -2 * a.eps, stream)
-            jb.jb_perturb(tab, s_own, a.eps, stream)
-            jb.jb_apply_updates(tab, seeds[t], q, a.lr, 1.0, a.qscale, stream)
+            jb.jb_perturb(tab, s_own, eps, stream)
+            jb.jb_perturb(tab, s_own, -2 * eps, stream)
+            jb.jb_perturb(tab, s_own, eps, stream)
+            jb.jb_apply_updates(tab, seeds, q, lr, 1.0, qscale, stream)
             done = torch.cuda.Event()
             done.record(stream)
-            s_out.wait_event(done)
-            with torch.cuda.stream(s_out):
-                host_bufs[gi].copy_(dev_bufs[gi], non_blocking=True)
-            out_done[gi] = torch.cuda.Event()
-            out_done[gi].record(s_out)
+            self.s_out.wait_event(done)
+            with torch.cuda.stream(self.s_out):
+                self.host_bufs[gi].copy_(self.dev_bufs[gi], non_blocking=True)
+            self.out_done[gi] = torch.cuda.Event()
+            self.out_done[gi].record(self.s_out)
+
+
+def run_e2e(a, jb, tensors, offs, seeds, codes, ghat, mids, own, stream, N, esize,
+            units_per_step, dist, n_groups=32):
+    """The step end to end (E2EPipeline), timed from the first copy in to the last
+    copy out, after one untimed step."""
+    import torch
+    pipe = E2EPipeline(jb, tensors, offs, stream, n_groups)
+
+    def step(t):
+        q = codes[t]
+        q[own] = jb.jb_quantize_grad(float(ghat[t]), a.qscale)
+        pipe.step((int(mids[own]), t, 0), seeds[t], q, a.eps, a.lr, a.qscale)
 
     base = a.warmup + a.steps
     step(base)
@@ -432,29 +450,30 @@ def run_e2e(a, jb, tensors, offs, seeds, codes, ghat, mids, own, stream, N, esiz
     if dist is not None:
         dist.barrier()
     x0, x1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    x0.record(s_in)
+    x0.record(pipe.s_in)
     for t in range(base + 1, base + 1 + a.e2e_steps):
         step(t)
-    x1.record(s_out)
+    x1.record(pipe.s_out)
     torch.cuda.synchronize()
     xms = x0.elapsed_time(x1) / a.e2e_steps
     # the same copies without overlap, for reference
     y0, y1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     y0.record(stream)
-    for h, d in zip(host_bufs, dev_bufs):
+    for h, d in zip(pipe.host_bufs, pipe.dev_bufs):
         d.copy_(h, non_blocking=True)
     y1.record(stream)
     z1 = torch.cuda.Event(enable_timing=True)
-    for h, d in zip(host_bufs, dev_bufs):
+    for h, d in zip(pipe.host_bufs, pipe.dev_bufs):
         h.copy_(d, non_blocking=True)
     z1.record(stream)
     torch.cuda.synchronize()
     h2d_ms, d2h_ms = y0.elapsed_time(y1), y1.elapsed_time(z1)
     xms, _ = aggregate_ranks(xms, 0.0, dist, torch.device("cuda", torch.cuda.current_device()))
-    del host_bufs, dev_bufs, views, tables
+    groups, copy_bytes = len(pipe.groups), pipe.copy_bytes
+    del pipe
     return {"value": units_per_step / (xms / 1e3), "unit": UNIT,
             "h2d_bytes_per_step": copy_bytes, "d2h_bytes_per_step": copy_bytes,
-            "ms_per_step": xms, "groups": len(groups), "h2d_ms": h2d_ms, "d2h_ms": d2h_ms}
+            "ms_per_step": xms, "groups": groups, "h2d_ms": h2d_ms, "d2h_ms": d2h_ms}
 
 
 # The sources the update kernel's device code and launch shape are built from.
