@@ -428,19 +428,29 @@ __device__ __forceinline__ void update_tile(const P& p, Tile<T, V>& tl) {
     add_acc<T, V, false>(tl, acc);
 }
 
-// theta <- fma(eps, z, theta) over the tile.
+// theta <- fma(eps, z, theta) over the tile. The Philox words of vector j + 1 are
+// computed while vector j is transformed, so the integer-multiply and fp32 work
+// of neighbouring vectors interleave (as the update does across seeds).
 template <typename T, int V, typename P>
 __device__ __forceinline__ void perturb_tile(const P& p, Tile<T, V>& tl) {
     constexpr int B = Traits<T>::E / 4;
     const SeedConst sc = seed_const(seed_key(p.seeds[0]));
     const float2 eps = splat(p.seeds[0].coef);
-    uint4 w[V][B];
-    tile_words<V, B>(sc, tl.blk, w);
+    uint4 wc[B], wn[B];
 #pragma unroll
-    for (int j = 0; j < V; ++j)
+    for (int b = 0; b < B; ++b)
+        wc[b] = philox_block(sc, static_cast<uint32_t>(tl.blk[0]) + b, static_cast<uint32_t>(tl.blk[0] >> 32));
+#pragma unroll
+    for (int j = 0; j < V; ++j) {
+        if (j + 1 < V) {
+#pragma unroll
+            for (int b = 0; b < B; ++b)
+                wn[b] = philox_block(sc, static_cast<uint32_t>(tl.blk[j + 1]) + b,
+                                     static_cast<uint32_t>(tl.blk[j + 1] >> 32));
+        }
 #pragma unroll
         for (int b = 0; b < B; ++b) {
-            const GaussPair g = box_muller2(w[j][b]);
+            const GaussPair g = box_muller2(wc[b]);
             const float2 ev = fma2<kPackO>(eps, g.even, make_float2(tl.x[j][4 * b + 0], tl.x[j][4 * b + 2]));
             const float2 od = fma2<kPackO>(eps, g.odd, make_float2(tl.x[j][4 * b + 1], tl.x[j][4 * b + 3]));
             tl.x[j][4 * b + 0] = ev.x;
@@ -448,6 +458,11 @@ __device__ __forceinline__ void perturb_tile(const P& p, Tile<T, V>& tl) {
             tl.x[j][4 * b + 1] = od.x;
             tl.x[j][4 * b + 3] = od.y;
         }
+        if (j + 1 < V) {
+#pragma unroll
+            for (int b = 0; b < B; ++b) wc[b] = wn[b];
+        }
+    }
 }
 
 template <typename T, bool UPDATE, typename P>
