@@ -361,7 +361,10 @@ __device__ __forceinline__ void visit_tiles(const P& p, bool also_src, Op&& op) 
 }
 
 // acc = sum_{k in [kb, ke)} c_k z_k for the tile, in fp32, in seed order (ke > kb).
-template <typename T, int V, typename P>
+// SINGLE_PIPE: a range of one seed computes the Philox words of vector j + 1 while
+// vector j is transformed (measured faster in the general update kernel, whose
+// replay groups are often one seed, and slower in the in-place one).
+template <typename T, int V, bool SINGLE_PIPE = false, typename P>
 __device__ __forceinline__ void accumulate_range(const P& p, const uint64_t (&blk)[V], uint32_t kb,
                                                  uint32_t ke, float2 (&acc)[V][Traits<T>::E / 4][2]) {
     constexpr int B = Traits<T>::E / 4;  // Philox blocks per vector
@@ -369,6 +372,36 @@ __device__ __forceinline__ void accumulate_range(const P& p, const uint64_t (&bl
     for (int j = 0; j < V; ++j)
 #pragma unroll
         for (int b = 0; b < B; ++b) acc[j][b][0] = acc[j][b][1] = make_float2(0.0f, 0.0f);
+    if constexpr (SINGLE_PIPE) {
+        if (ke - kb == 1) {
+            const SeedConst sc = seed_const(seed_key(p.seeds[kb]));
+            const float c = p.seeds[kb].coef;
+            uint4 wc[B], wn[B];
+#pragma unroll
+            for (int b = 0; b < B; ++b)
+                wc[b] = philox_block(sc, static_cast<uint32_t>(blk[0]) + b, static_cast<uint32_t>(blk[0] >> 32));
+#pragma unroll
+            for (int j = 0; j < V; ++j) {
+                if (j + 1 < V) {
+#pragma unroll
+                    for (int b = 0; b < B; ++b)
+                        wn[b] = philox_block(sc, static_cast<uint32_t>(blk[j + 1]) + b,
+                                             static_cast<uint32_t>(blk[j + 1] >> 32));
+                }
+#pragma unroll
+                for (int b = 0; b < B; ++b) {
+                    const GaussPair g = box_muller2(wc[b]);
+                    acc[j][b][0] = fma2<kPackO>(splat(c), g.even, acc[j][b][0]);
+                    acc[j][b][1] = fma2<kPackO>(splat(c), g.odd, acc[j][b][1]);
+                }
+                if (j + 1 < V) {
+#pragma unroll
+                    for (int b = 0; b < B; ++b) wc[b] = wn[b];
+                }
+            }
+            return;
+        }
+    }
     if constexpr (Traits<T>::PIPE) {
         // Philox words of seed k + 1 are computed while seed k is transformed and
         // accumulated: the integer-multiply work and the fp32 work are independent
@@ -492,7 +525,7 @@ __global__ void __launch_bounds__(kThreads) general_update_kernel(const __grid_c
         for (uint32_t g = 0; g < p.n_groups; ++g) {
             const uint32_t ke = p.group_end[g];  // > kb: the host drops empty groups
             float2 acc[V][Traits<T>::E / 4][2];
-            accumulate_range<T, V>(p, tl.blk, kb, ke, acc);
+            accumulate_range<T, V, true>(p, tl.blk, kb, ke, acc);
             add_acc<T, V, true>(tl, acc);
             kb = ke;
         }
