@@ -64,10 +64,10 @@ namespace {
 #define JB_SU_BF16 4
 #endif
 #ifndef JB_SG_F32  // warp tiles per span, general update kernel
-#define JB_SG_F32 1
+#define JB_SG_F32 4
 #endif
 #ifndef JB_SG_BF16
-#define JB_SG_BF16 1
+#define JB_SG_BF16 4
 #endif
 #ifndef JB_SP_F32  // warp tiles per span, perturb kernel
 #define JB_SP_F32 4
@@ -526,7 +526,10 @@ __global__ void __launch_bounds__(kThreads) general_update_kernel(const __grid_c
             const uint32_t ke = p.group_end[g];  // > kb: the host drops empty groups
             float2 acc[V][Traits<T>::E / 4][2];
             accumulate_range<T, V, true>(p, tl.blk, kb, ke, acc);
-            add_acc<T, V, true>(tl, acc);
+            // the store rounds the last group's sum to T; rounding twice to the
+            // nearest gives the same bits, so only earlier groups round here
+            if (g + 1 < p.n_groups) add_acc<T, V, true>(tl, acc);
+            else add_acc<T, V, false>(tl, acc);
             kb = ke;
         }
     });
