@@ -112,17 +112,19 @@ __global__ void __launch_bounds__(kThreadsQ4) q4_perturb_kernel(const __grid_con
         const float sc_in = any ? scale[u >> 2] : 0.0f;
 
         // dequantize and perturb
+        // the Philox words of block b + 1 are computed while block b is transformed
         float w[16];
-        uint4 words[4];
         const uint64_t blk0 = (g.fo + static_cast<uint64_t>(i0)) >> 2;  // fo % 4 == 0
-#pragma unroll
-        for (int b = 0; b < 4; ++b)
-            words[b] = philox_block(sc, static_cast<uint32_t>(blk0 + b),
-                                    static_cast<uint32_t>((blk0 + b) >> 32));
         float m = 0.0f;
+        uint4 wcur = philox_block(sc, static_cast<uint32_t>(blk0), static_cast<uint32_t>(blk0 >> 32));
 #pragma unroll
         for (int b = 0; b < 4; ++b) {
-            const GaussPair z = box_muller2(words[b]);
+            uint4 wnext;
+            if (b + 1 < 4)
+                wnext = philox_block(sc, static_cast<uint32_t>(blk0 + b + 1),
+                                     static_cast<uint32_t>((blk0 + b + 1) >> 32));
+            const GaussPair z = box_muller2(wcur);
+            if (b + 1 < 4) wcur = wnext;
             const float zz[4] = {z.even.x, z.odd.x, z.even.y, z.odd.y};
 #pragma unroll
             for (int t = 0; t < 4; ++t) {
