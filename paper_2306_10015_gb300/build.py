@@ -43,8 +43,10 @@ def build(force: bool = False, verbose: bool = False) -> str:
     if not force and not _stale():
         return LIB
     os.makedirs(OUT_DIR, exist_ok=True)
+    # no implicit a * b + c -> fma contraction on either side: every rounding in
+    # the device code is the one its intrinsic names
     common = ARCH + ["-O3", "-std=c++17", "-lineinfo", "-I", INCLUDE, "-I", CSRC,
-                     "-Xcompiler", "-fPIC,-fvisibility=hidden,-ffp-contract=off",
+                     "--fmad=false", "-Xcompiler", "-fPIC,-fvisibility=hidden,-ffp-contract=off",
                      "--expt-relaxed-constexpr"]
     if verbose:
         common += ["-Xptxas", "-v"]
