@@ -16,7 +16,7 @@
 namespace jb {
 
 #ifndef JB_THREADS
-#define JB_THREADS 256
+#define JB_THREADS 512
 #endif
 constexpr int kThreads = JB_THREADS;   // threads per CTA
 constexpr int kMaxSeedsPerLaunch = 512;
