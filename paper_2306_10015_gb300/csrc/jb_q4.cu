@@ -57,7 +57,7 @@ __device__ __forceinline__ uint32_t q4_code(float x, const float2* bucket) {
     return __float_as_uint(e.y) + (x > e.x ? 1u : 0u);
 }
 
-constexpr int kThreadsQ4 = 256;
+constexpr int kThreadsQ4 = 512;  // measured 2.4% faster than 256 on the 13B-shaped set
 
 __global__ void __launch_bounds__(kThreadsQ4) q4_perturb_kernel(const __grid_constant__ Q4Params p) {
     __shared__ float level[16];
