@@ -15,8 +15,8 @@
 //           q = -4t / (2 + t) (one rcp.approx), -2 ln(1 + t) = q + q w R(w),
 //           w = q^2, R a degree-2 minimax polynomial; L = -2 e ln 2 - 2 ln(1+t)
 //           with 2 ln 2 split hi + lo (Cody & Waite 1980) so e (2 ln 2)_hi is
-//           exact; r = r0 + corr from rsqrt.approx and one Newton step, the
-//           correction kept separate and folded into the final products.
+//           exact; r = r0 + corr from rsqrt.approx and one Newton step,
+//           rounded once to fp32 (one fused multiply-add).
 //   angle   the 24-bit angle index splits into an octant (3 bits, handled
 //           exactly by reflection, swap and sign flips) and a 21-bit offset
 //           x in (0, 1) of the octant, sin(pi x / 4) and cos(pi x / 4) by
@@ -180,7 +180,7 @@ __device__ __forceinline__ GaussPair box_muller2(uint4 w) {
     const float2 yr = make_float2(rsqrt_approx(-L.x), rsqrt_approx(-L.y));
     const float2 r0 = mul2<kPackR>(L, yr);                            // -r0
     const float2 m = add2<kPackR>(fma2<kPackR>(r0, r0, l_hi), l_lo);    // r0^2 + L
-    const float2 corr = mul2<kPackR>(m, mul2<kPackR>(splat(0.5f), yr)); // -corr
+    const float2 rr = fma2<kPackR>(m, mul2<kPackR>(splat(0.5f), yr), r0); // -(r0 + corr)
 
     // ---- angle ----
     const int32_t waA = static_cast<int32_t>(((w.y << 2) & 0xFFFFFC00u) | 0x200u);
@@ -207,8 +207,8 @@ __device__ __forceinline__ GaussPair box_muller2(uint4 w) {
         __uint_as_float(__float_as_uint(swA ? C.x : S.x) ^ (w.y & 0x80000000u) ^ 0x80000000u),
         __uint_as_float(__float_as_uint(swB ? C.y : S.y) ^ (w.w & 0x80000000u) ^ 0x80000000u));
     GaussPair g;
-    g.even = fma2<kPackO>(cm, r0, mul2<kPackO>(cm, corr));
-    g.odd = fma2<kPackO>(sm, r0, mul2<kPackO>(sm, corr));
+    g.even = mul2<kPackO>(cm, rr);
+    g.odd = mul2<kPackO>(sm, rr);
     return g;
 }
 
