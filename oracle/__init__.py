@@ -93,6 +93,9 @@ def lib() -> ctypes.CDLL:
             L.jbo_update_delta_at.argtypes = [vp, u64, vp, vp, ctypes.c_int, ctypes.c_double,
                                               ctypes.c_double, ctypes.c_double, vp]
             L.jbo_update_delta_at.restype = ctypes.c_int
+            L.jbo_update_delta_abs_at.argtypes = [vp, u64, vp, vp, ctypes.c_int, ctypes.c_double,
+                                                  ctypes.c_double, ctypes.c_double, vp, vp]
+            L.jbo_update_delta_abs_at.restype = ctypes.c_int
             L.jbo_q4_levels.argtypes = [vp]
             L.jbo_q4_quantize.argtypes = [vp, u64, vp, vp]
             L.jbo_q4_dequantize.argtypes = [vp, vp, u64, vp]
@@ -276,6 +279,20 @@ def update_delta_at(idx: np.ndarray, seeds, q, lr: float, denom: float,
     _check(lib().jbo_update_delta_at(_ptr(i), i.size, _ptr(s), _ptr(qa), len(s), lr, denom,
                                      qscale, _ptr(out)))
     return out
+
+
+def update_delta_abs_at(idx: np.ndarray, seeds, q, lr: float, denom: float,
+                        qscale: float) -> tuple:
+    """(sum_k c_k z_k, sum_k |c_k z_k|) at global indices idx, in double; the first
+    is update_delta_at's value bit for bit."""
+    i = np.ascontiguousarray(idx, dtype=np.uint64)
+    s = seeds_array(seeds)
+    qa = np.ascontiguousarray(q, dtype=np.int8)
+    out = np.empty(i.size, dtype=np.float64)
+    mag = np.empty(i.size, dtype=np.float64)
+    _check(lib().jbo_update_delta_abs_at(_ptr(i), i.size, _ptr(s), _ptr(qa), len(s), lr, denom,
+                                         qscale, _ptr(out), _ptr(mag)))
+    return out, mag
 
 
 # --- 4-bit weights -----------------------------------------------------------

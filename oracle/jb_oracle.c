@@ -321,6 +321,32 @@ int jbo_update_delta_at(const uint64_t* idx, uint64_t n, const jbo_seed* seeds, 
     return rc;
 }
 
+/* The same sum together with sum_k |c_k z_k(e)| (the size of the operands,
+ * which the parity tolerances scale with), from one evaluation of each z. */
+int jbo_update_delta_abs_at(const uint64_t* idx, uint64_t n, const jbo_seed* seeds,
+                            const int8_t* q, int K, double lr, double denom, double qscale,
+                            double* out, double* out_abs) {
+    jbo_seed* ss = (jbo_seed*)malloc(sizeof(jbo_seed) * (size_t)(K > 0 ? K : 1));
+    double* cc = (double*)malloc(sizeof(double) * (size_t)(K > 0 ? K : 1));
+    if (!ss || !cc) { free(ss); free(cc); return -2; }
+    int rc = prepare_update(seeds, q, K, lr, denom, qscale, ss, cc);
+    if (rc == 0) {
+        #pragma omp parallel for schedule(static)
+        for (int64_t j = 0; j < (int64_t)n; ++j) {
+            double acc = 0.0, mag = 0.0;
+            for (int k = 0; k < K; ++k) {
+                const double t = cc[k] * jbo_gaussian(ss[k], idx[j]);
+                acc += t;
+                mag += fabs(t);
+            }
+            out[j] = acc;
+            out_abs[j] = mag;
+        }
+    }
+    free(ss); free(cc);
+    return rc;
+}
+
 /* ------------------------------------------------------------------------ */
 /* 4-bit weights (Section 3, Training Speed: weights are dequantized before   */
 /* the noise is added and quantized again). Reading (the paper fixes no       */

@@ -52,6 +52,9 @@ int jbo_update_at(const void* in, void* out, int dtype, const uint64_t* idx, uin
                   double qscale);
 int jbo_update_delta_at(const uint64_t* idx, uint64_t n, const jbo_seed* seeds, const int8_t* q,
                         int K, double lr, double denom, double qscale, double* out);
+int jbo_update_delta_abs_at(const uint64_t* idx, uint64_t n, const jbo_seed* seeds,
+                            const int8_t* q, int K, double lr, double denom, double qscale,
+                            double* out, double* out_abs);
 
 void jbo_q4_levels(float out[16]);
 void jbo_q4_quantize(const double* w, uint64_t n, uint8_t* codes, float* scale);

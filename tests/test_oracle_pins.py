@@ -361,6 +361,24 @@ def test_update_is_linear_in_pairs():
                                    c * oracle.gaussian_at(s[k], idx), rtol=1e-15)
 
 
+def test_update_delta_abs_is_delta_and_magnitude():
+    """The one-pass (sum c z, sum |c z|) helper: its sum is update_delta_at's bit for
+    bit, and update_at is the storage rounding of theta + that sum; its magnitude is
+    sum_k |c_k| |z_k| term by term."""
+    idx = np.array([0, 1, 2, 3, 5, 1 << 33, (1 << 34) + 7, 123456789], dtype=np.uint64)
+    s = _seeds(6)
+    q = np.array([3, -100, 127, -128, 0, 64], dtype=np.int8)
+    delta, mag = oracle.update_delta_abs_at(idx, s, q, 1e-3, 6.0, 8.0)
+    assert np.array_equal(delta, oracle.update_delta_at(idx, s, q, 1e-3, 6.0, 8.0))
+    want = sum(abs(oracle.coefficient(q[k], 1e-3, 6.0, 8.0)) * np.abs(oracle.gaussian_at(s[k], idx))
+               for k in range(6))
+    np.testing.assert_allclose(mag, want, rtol=1e-14)
+    assert np.all(mag >= np.abs(delta))
+    th = oracle.round_bf16(synthetic.normal_values(idx.size, 0.02, 8).astype(np.float64))
+    assert np.array_equal(oracle.update_at(th, idx, s, q, 1e-3, 6.0, 8.0),
+                          oracle.round_bf16(oracle.bf16_to_f64(th) + delta))
+
+
 def test_update_at_matches_contiguous():
     th = synthetic.normal_values(4096, 0.02, 6)
     hb = oracle.round_bf16(th.astype(np.float64))
