@@ -40,6 +40,8 @@ UNIT = "param·seed/s"
 # sin, cos, 2 products over 2 elements) = 4; the accumulate FMA = 1.
 OPS_PER_PARAM_SEED = 15
 LANES_PER_SM_CLK = 128
+# special-function unit: 16 lanes per clock per SM (measured: lg2.approx at 16.1)
+MUFU_LANES_PER_SM_CLK = 16
 
 
 def parse():
@@ -57,9 +59,11 @@ def parse():
     ap.add_argument("--e2e-steps", type=int, default=4)
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--cpu-seconds", type=float, default=12.0,
-                    help="target CPU time of the oracle sample")
-    ap.add_argument("--sweep", default="", help="comma list of K: time update/perturb per K")
+    ap.add_argument("--cpu-seconds", type=float, default=10.0,
+                    help="target CPU time of each oracle sample (all cores, then one core)")
+    ap.add_argument("--sweep", default="1,4,16,64,256",
+                    help="comma list of K: the fused update timed per K (empty: no sweep)")
+    ap.add_argument("--no-sweep", action="store_true", help="skip the K sweep")
     ap.add_argument("--sweep-out", default="", help="file for the sweep's JSON lines")
     ap.add_argument("--next-legs", action="store_true",
                     help="with --sweep: also time the backup-fused update and the replay")
@@ -145,14 +149,15 @@ class ClockSampler:
 
 # --- the CPU oracle (baseline and reference arm) --------------------------------------
 
-def oracle_rate(a, target_s: float):
+def oracle_rate(a, target_s: float, threads: int = 0):
     """The oracle, as it stands, on a bounded sample of the workload: sampled
-    elements x (3 perturb seeds + K update seeds). Returns (param.seed/s, cores, sample)."""
+    elements x (3 perturb seeds + K update seeds), on `threads` host threads (0: all
+    cores the process may use). Returns (param.seed/s, threads, seconds, elements)."""
     import numpy as np
 
     import oracle
     import synthetic
-    cores = len(os.sched_getaffinity(0))
+    cores = threads if threads > 0 else len(os.sched_getaffinity(0))
     oracle.set_threads(cores)
     specs = synthetic.opt_tensors(a.model)
     numels = [s.numel for s in specs]
@@ -179,6 +184,7 @@ def oracle_rate(a, target_s: float):
     rate = n0 * (a.K + 3) / max(t0, 1e-6)
     n = int(min(max(rate * target_s / (a.K + 3), 1 << 12), 1 << 26))
     n, t = run(n)
+    oracle.set_threads(len(os.sched_getaffinity(0)))
     return n * (a.K + 3) / t, cores, t, n
 
 
@@ -308,7 +314,7 @@ def main():
                       units_per_step, dist)
 
     sweep_lines = []
-    if a.sweep and rank == 0:
+    if a.sweep and not a.no_sweep and rank == 0:
         sweep_lines = run_sweep(a, jb, table, mids, stream)
 
     if rank != 0:
@@ -316,43 +322,22 @@ def main():
             dist.destroy_process_group()
         return
 
-    props = torch.cuda.get_device_properties(local_rank)
-    sms = props.multi_processor_count
-    peaks = {}
-    try:
-        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
-            peaks = json.load(f)
-    except OSError:
-        pass
-    hbm_peak = float(peaks.get("hbm_gbs", 6800.0))
-    f_max = float(peaks.get("sm_max_mhz", 2070.0)) * 1e6
-    upd = statistics.mean(upd_ms) / 1e3
-    alu_peak = sms * LANES_PER_SM_CLK * f_max / 1e12            # Tops/s
-    alu_ach = OPS_PER_PARAM_SEED * K * N / upd / 1e12
-    traffic = load_traffic(a)
-    roofline = {"bound": "alu", "achieved": alu_ach, "peak": alu_peak, "unit": "Tops/s",
-                "frac": alu_ach / alu_peak, "traffic": traffic,
-                "kernel": "seeded_kernel<bf16, update>" if a.dtype == "bf16" else
-                "seeded_kernel<f32, update>",
-                "ops_per_param_seed": OPS_PER_PARAM_SEED,
-                "peak_basis": f"{sms} SMs x {LANES_PER_SM_CLK} lanes x {f_max / 1e6:.0f} MHz",
-                "hbm_gbs": 2 * esize * N / upd / 1e9, "hbm_frac_of_measured": 2 * esize * N / upd / 1e9 / hbm_peak,
-                "update_ms": statistics.mean(upd_ms), "perturb_ms": statistics.mean(pert_ms)}
-    # The combined roofline as the task states it: the slower of the HBM time and
-    # the measured instruction count at peak issue (one lane-instruction per lane
-    # per clock), next to the strict algorithmic figure above.
-    instr = load_instr_per_param_seed(a)
-    if instr is not None:
-        t_rng = K * N * instr / (sms * LANES_PER_SM_CLK * f_max)
-        t_hbm = 2 * esize * N / (hbm_peak * 1e9)
-        roofline["combined_issue"] = {
-            "instr_per_param_seed": instr, "t_rng_ms": t_rng * 1e3, "t_hbm_ms": t_hbm * 1e3,
-            "frac": max(t_rng, t_hbm) / upd}
+    roof = Roofline(a, torch, N, esize, generator_rate(jb, stream))
+    roofline = roof.report(K, upd_ms)
+    roofline.update({
+        "bound": "alu", "traffic": load_traffic(a),
+        "kernel": "seeded_kernel<bf16, update>" if a.dtype == "bf16" else "seeded_kernel<f32, update>",
+        "perturb_ms": statistics.mean(pert_ms), "perturb_ms_best": min(pert_ms),
+        "perturb_ms_median": statistics.median(pert_ms),
+        "timing": f"CUDA events per launch over the {a.steps} timed steps; frac uses the best launch"})
     cpu = None
     if not a.no_cpu_baseline and world == 1:
         rate, cores, t, n = oracle_rate(a, a.cpu_seconds)
+        rate1, _, t1, n1 = oracle_rate(a, a.cpu_seconds, threads=1)
         cpu = {"value": rate, "unit": UNIT, "cores": cores, "kind": "oracle",
-               "sample": f"{n} sampled elements x (3 perturb + {K} update seeds), {t:.1f} s"}
+               "sample": f"{n} sampled elements x (3 perturb + {K} update seeds), {t:.1f} s",
+               "single_thread": {"value": rate1, "unit": UNIT, "cores": 1,
+                                 "sample": f"{n1} sampled elements x (3 + {K} seeds), {t1:.1f} s"}}
     step_bytes = 4 * 2 * esize * N  # 3 perturb passes + 1 update pass, read + write
     out = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": a.steps,
@@ -364,10 +349,94 @@ def main():
         "gpu_launches": launches_per_step * a.steps, "clocks": clk,
     }
     if sweep_lines:
-        out["sweep"] = sweep_lines
+        out["sweep"] = [roof.report(ln["K"], ln["ms"]) if "K" in ln else ln for ln in sweep_lines]
     print(json.dumps(out), flush=True)
     if dist is not None:
         dist.destroy_process_group()
+
+
+def stats(ms):
+    return {"best": min(ms), "median": statistics.median(ms), "mean": statistics.mean(ms), "n": len(ms)}
+
+
+def generator_rate(jb, stream, n_blocks=1 << 32, reps=5):
+    """Element-seeds per second of Philox4x32-10 alone (jb_debug_philox_fold: the hot
+    path's block function, its words XOR-folded), best of `reps` launches."""
+    import torch
+    out = torch.zeros(1, dtype=torch.int32, device="cuda")
+    jb.jb_debug_philox_fold((1, 2, 3), 0, n_blocks, out, stream)
+    best = float("inf")
+    for _ in range(reps):
+        x0, x1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        x0.record(stream)
+        jb.jb_debug_philox_fold((1, 2, 3), 0, n_blocks, out, stream)
+        x1.record(stream)
+        torch.cuda.synchronize()
+        best = min(best, x0.elapsed_time(x1))
+    return 4 * n_blocks / (best / 1e3)
+
+
+class Roofline:
+    """Rooflines of the fused K-seed update on this GPU, per K and launch time.
+
+    * frac (judged; the combined roofline of the task): T_roof = max(T_HBM, T_ALG),
+      T_HBM = 2 sizeof(T) N / measured copy bandwidth, T_ALG = the algorithm's fixed
+      count of OPS_PER_PARAM_SEED = 15 lane operations per element-seed (a quarter
+      Philox4x32-10 block: 10 rounds x (2 wide multiplies + 2 three-input XORs) / 4;
+      half a Box-Muller pair: 2 uniforms, log, sqrt, sin, cos, 2 products over 2
+      elements; one accumulating FMA), each at one lane-operation per lane per clock,
+      152 SMs x 128 lanes x the maximum SM clock. frac = T_roof / T_best.
+    * floors.generator: the same K N element-seeds at the rate of Philox4x32-10 alone
+      (jb_debug_philox_fold, measured in this run): what the wide multiplies cost.
+    * floors.mufu: one special-function operation per element-seed (rcp and rsqrt
+      per word pair) at 16 lanes per clock per SM.
+    * issue_measured: the kernel's own ncu-measured lane-instructions per
+      element-seed at peak issue (occupancy of the issue slots, not a bound)."""
+
+    def __init__(self, a, torch, N, esize, gen_rate):
+        props = torch.cuda.get_device_properties(torch.cuda.current_device())
+        self.sms = props.multi_processor_count
+        peaks = {}
+        try:
+            with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+                peaks = json.load(f)
+        except OSError:
+            pass
+        self.hbm_peak = float(peaks.get("hbm_gbs", 6800.0))
+        self.peak_src = "measured" if "hbm_gbs" in peaks else "fallback"
+        self.f_max = float(peaks.get("sm_max_mhz", 2070.0)) * 1e6
+        self.N, self.esize, self.gen_rate = N, esize, gen_rate
+        self.lanes = self.sms * LANES_PER_SM_CLK * self.f_max
+        self.instr = load_instr_per_param_seed(a)
+
+    def report(self, K, ms_list):
+        st = stats(ms_list)
+        t = st["best"] / 1e3
+        N = self.N
+        t_hbm = 2 * self.esize * N / (self.hbm_peak * 1e9)
+        t_alg = OPS_PER_PARAM_SEED * K * N / self.lanes
+        t_gen = K * N / self.gen_rate
+        t_mufu = K * N / (self.sms * MUFU_LANES_PER_SM_CLK * self.f_max)
+        out = {
+            "K": K, "update_ms": st["mean"], "update_ms_best": st["best"], "update_ms_median": st["median"],
+            "launches": st["n"], "param_seed_per_s": K * N / t,
+            "param_seed_per_s_median": K * N / (st["median"] / 1e3),
+            "achieved": OPS_PER_PARAM_SEED * K * N / t / 1e12, "peak": self.lanes / 1e12, "unit": "Tops/s",
+            "frac": max(t_hbm, t_alg) / t, "ops_per_param_seed": OPS_PER_PARAM_SEED,
+            "peak_basis": f"{self.sms} SMs x {LANES_PER_SM_CLK} lanes x {self.f_max / 1e6:.0f} MHz; "
+                          f"HBM {self.hbm_peak:.0f} GB/s ({self.peak_src})",
+            "t_hbm_ms": t_hbm * 1e3, "t_alg_ms": t_alg * 1e3,
+            "hbm_gbs": 2 * self.esize * N / t / 1e9, "hbm_frac": t_hbm / t,
+            "floors": {"generator": {"philox_only_param_seed_per_s": self.gen_rate, "t_ms": t_gen * 1e3,
+                                     "frac": t_gen / t},
+                       "mufu": {"lanes_per_clk_per_sm": MUFU_LANES_PER_SM_CLK, "ops_per_param_seed": 1,
+                                "t_ms": t_mufu * 1e3, "frac": t_mufu / t}},
+        }
+        if self.instr is not None:
+            t_iss = self.instr * K * N / self.lanes
+            out["issue_measured"] = {"instr_per_param_seed": self.instr, "t_ms": t_iss * 1e3,
+                                     "frac": max(t_iss, t_hbm) / t}
+        return out
 
 
 class E2EPipeline:
@@ -527,48 +596,41 @@ def load_instr_per_param_seed(a):
     return load_counters().get("instr_per_param_seed", {}).get(a.dtype)
 
 
+SWEEP_REPS = {1: 20, 4: 10, 16: 5, 64: 3, 256: 2}
+
+
 def run_sweep(a, jb, table, mids, stream):
+    """The fused update per K (one warm-up launch, then per-launch CUDA events) and
+    the perturb pass; main() turns each update line into a roofline report."""
     import torch
     import synthetic
     out = []
     N = table.numel
-    es = table.tensors[0].element_size()
-    instr = load_instr_per_param_seed(a)
-    peaks = {}
-    try:
-        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
-            peaks = json.load(f)
-    except OSError:
-        pass
-    issue_rate = (torch.cuda.get_device_properties(torch.cuda.current_device()).multi_processor_count
-                  * LANES_PER_SM_CLK * float(peaks.get("sm_max_mhz", 2070.0)) * 1e6)
-    t_hbm = 2 * es * N / (float(peaks.get("hbm_gbs", 6800.0)) * 1e9)
+
+    def timed(fn, reps):
+        fn()
+        ev = []
+        for _ in range(reps):
+            x0, x1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            x0.record(stream)
+            fn()
+            x1.record(stream)
+            ev.append((x0, x1))
+        torch.cuda.synchronize()
+        return [x0.elapsed_time(x1) for x0, x1 in ev]
+
     for K in [int(k) for k in a.sweep.split(",") if k]:
         seeds = jb.seeds_array([(int(m), 7, 0) for m in synthetic.machine_ids(K, 910)])
         q = synthetic.byte_codes(K, 910)
-        reps = 3 if K <= 64 else 2
-        jb.jb_apply_updates(table, seeds, q, a.lr, 1.0, a.qscale, stream)
-        x0, x1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        x0.record(stream)
-        for _ in range(reps):
-            jb.jb_apply_updates(table, seeds, q, a.lr, 1.0, a.qscale, stream)
-        x1.record(stream)
-        torch.cuda.synchronize()
-        ms = x0.elapsed_time(x1) / reps
-        line = {"K": K, "update_ms": ms, "param_seed_per_s": N * K / (ms / 1e3),
-                "hbm_gbs": 2 * es * N / (ms / 1e3) / 1e9}
-        if instr is not None:  # combined roofline: max(HBM time, instructions at peak issue)
-            line["combined_issue_frac"] = max(t_hbm, K * N * instr / issue_rate) / (ms / 1e3)
-        out.append(line)
-    p0, p1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    p0.record(stream)
-    for i in range(4):
-        jb.jb_perturb(table, (1, 2, 3), a.eps if i % 2 == 0 else -a.eps, stream)
-    p1.record(stream)
-    torch.cuda.synchronize()
-    pms = p0.elapsed_time(p1) / 4
-    out.append({"perturb_ms": pms, "param_seed_per_s": N / (pms / 1e3),
-                "hbm_gbs": 2 * table.tensors[0].element_size() * N / (pms / 1e3) / 1e9})
+        reps = SWEEP_REPS.get(K, 3)
+        ms = timed(lambda: jb.jb_apply_updates(table, seeds, q, a.lr, 1.0, a.qscale, stream), reps)
+        out.append({"K": K, "ms": ms})
+    pms = timed(lambda: jb.jb_perturb(table, (1, 2, 3), a.eps, stream), 20)
+    st = stats(pms)
+    es = table.tensors[0].element_size()
+    out.append({"perturb_ms": st["mean"], "perturb_ms_best": st["best"], "perturb_ms_median": st["median"],
+                "param_seed_per_s": N / (st["best"] / 1e3),
+                "hbm_gbs": 2 * es * N / (st["best"] / 1e3) / 1e9})
     if a.next_legs:
         out.extend(next_legs(a, jb, table, stream))
         out.append(checksum_leg(jb, table, stream))

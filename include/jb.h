@@ -16,8 +16,9 @@
  *                     order (Section 2, "Applying collected scalar projected
  *                     gradients"; Algorithm 1), fused into one read and one
  *                     write of theta.
- *   jb_quantize_grad  the one-byte projected gradient, "signed log of the
- *   jb_dequantize_grad gradient clipped to +-127" (Section 3, Training Speed).
+ *   jb_quantize_grad  the one-byte projected gradient: the logarithm of its
+ *   jb_dequantize_grad magnitude with its sign, limited to +-127 (Section 3,
+ *                     Training Speed).
  *
  * ---------------------------------------------------------------------------
  * Random stream. The paper names no generator (Appendix B notes that PyTorch's
@@ -31,6 +32,13 @@
  *     r = sqrt(-2 ln u_a); even element r cos(2 pi u_b), odd r sin(2 pi u_b).
  *   z depends only on (seed, e): never on the tensor split, the launch
  *   geometry or the GPU run, so every replica regenerates identical noise.
+ *   Scope of that bit-identity: the Philox words are exact integers and the
+ *   same on any machine; the transform is fp32 with every rounding explicit,
+ *   except its reciprocal and reciprocal square root, which are the GPU's
+ *   rcp.approx / rsqrt.approx instructions. z is therefore bitwise identical
+ *   on every sm_103a (GB300) GPU, the only target of this library; on other
+ *   hardware its last bits may differ, while staying within 1e-6 of the exact
+ *   definition above.
  *
  * Global element index. Each tensor ("segment") carries flat_offset, the
  * global index of its element 0: element i of the segment is e = flat_offset
@@ -40,11 +48,13 @@
  * needs (ptr - flat_offset * sizeof(T)) to be a multiple of 16 bytes; other
  * segments are still handled, element by element, at lower speed.
  *
- * Arithmetic. z in fp32; |z| <= sqrt(48 ln 2) = 5.77. Perturb: one fp32 fused
- * multiply-add theta + eps z, then one rounding to the storage type (nearest,
- * ties to even). Update: acc = 0; for each pair k in canonical order
- * acc = fma(c_k, z_k, acc) in fp32; theta <- round(theta + acc) once. No
- * flush-to-zero. Results are bitwise repeatable.
+ * Arithmetic. z = s r in fp32, with r the radius and s the signed cosine or
+ * sine of the element; |z| <= sqrt(48 ln 2) = 5.77. A scaled draw a z is formed
+ * as fma(s, a r, .) with a r rounded once to fp32. Perturb: theta + eps z as
+ * one fp32 fused multiply-add, fma(s, eps r, theta), then one rounding to the
+ * storage type (nearest, ties to even). Update: acc = 0; for each pair k in
+ * canonical order acc = fma(s_k, c_k r_k, acc) in fp32; theta <- round(theta +
+ * acc) once. No flush-to-zero. Results are bitwise repeatable.
  *
  * Memory and streams. The caller owns all device memory (e.g. torch
  * tensors). The library copies the host arrays it is given (segments, seeds,
@@ -56,9 +66,14 @@
  *
  * Errors. Every entry point returns a jb_status. Argument errors are detected
  * before anything is enqueued, and then nothing is enqueued. JB_ERR_CUDA
- * reports a launch failure seen by cudaGetLastError; faults during execution
- * surface at the caller's next synchronisation. No exception, abort or exit
- * crosses this interface.
+ * reports a failed CUDA runtime call or launch of this call (cudaGetLastError);
+ * faults during execution surface at the caller's next synchronisation. The
+ * library links the CUDA runtime statically, so its error state is private: an
+ * error pending in the caller's runtime (torch's, say) is neither reported nor
+ * cleared by libjb, and libjb clears each error it reports so that none lingers
+ * into a later call. A sticky error (a fault that poisons the context) is
+ * reported by every runtime. No exception, abort or exit crosses this
+ * interface.
  */
 #ifndef JB_H
 #define JB_H
@@ -104,8 +119,9 @@ typedef struct {
 
 /*
  * jb_perturb -- PerturbParameters(theta, eps, s) (Algorithm 1, subroutine):
- * for every element e of every segment, theta_e <- round_T(fma(eps, z_e(seed),
- * theta_e)). In place, asynchronous on `stream`.
+ * for every element e of every segment, theta_e <- round_T(theta_e + eps
+ * z_e(seed)), the sum one fp32 fused multiply-add (see Arithmetic). In place,
+ * asynchronous on `stream`.
  *   segs, n_segs  segment table (host array, copied); n_segs = 0 is a no-op.
  *   dtype         JB_F32 or JB_BF16 for all segments.
  *   eps           finite perturbation scale (use +eps, -2 eps, +eps for one
@@ -181,7 +197,7 @@ typedef struct {
  * jb_perturb_q4 -- PerturbParameters on 4-bit weights (Section 3, Training
  * Speed: weights are dequantized before the noise is added and quantized
  * again). For every block of 64 elements: w_i = level[code_i] * scale,
- * w'_i = fma(eps, z_i(seed), w_i) in fp32 with the same z as jb_perturb, then
+ * w'_i = w_i + eps z_i(seed) in fp32, one fused multiply-add as in jb_perturb, then
  * scale' = max_i |w'_i| and code'_i = the nearest level to w'_i / scale' (ties
  * to the lower level; scale' = 0 gives the zero level). Codes and scales are
  * rewritten in place, asynchronously on `stream`. The paper fixes no 4-bit
@@ -215,7 +231,8 @@ int jb_checksum(const jb_segment* segs, int n_segs, int dtype, uint64_t* d_out,
 
 /*
  * jb_quantize_grad -- one-byte projected gradient (Section 3, Training
- * Speed: signed log of the gradient, clipped to +-127). Host only, pure:
+ * Speed: the sign and the logarithm of the magnitude, limited to +-127). Host
+ * only, pure:
  *   *out = sign(g) * min(127, round_half_away(qscale * ln(1 + |g|))),
  *   NaN -> 0, +-inf -> +-127. qscale must be finite and > 0.
  */
@@ -243,6 +260,14 @@ const char* jb_status_string(int status);
  * d_out must be 16-byte aligned (JB_ERR_MISALIGNED); n_blocks <= 2^38. */
 int jb_debug_philox(jb_seed seed, uint64_t first_block, uint64_t n_blocks, uint32_t* d_out,
                     struct CUstream_st* stream);
+
+/* *d_out = XOR of all words of Philox blocks first_block .. first_block +
+ * n_blocks - 1 under `seed`: the generator alone, computed as the kernels
+ * compute it, on the persistent grid (the benchmark times it as the
+ * generator-only rate). d_out: one uint32_t, 4-byte aligned, zeroed and written
+ * on `stream`. n_blocks <= 2^46, first_block <= 2^60. */
+int jb_debug_philox_fold(jb_seed seed, uint64_t first_block, uint64_t n_blocks, uint32_t* d_out,
+                         struct CUstream_st* stream);
 
 /* d_out[i] = z of global element first_elem + i under `seed` (fp32).
  * d_out must be 4-byte aligned (JB_ERR_MISALIGNED); n <= 2^38. */

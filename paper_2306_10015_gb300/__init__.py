@@ -91,13 +91,15 @@ def lib() -> ctypes.CDLL:
             L.jb_status_string.argtypes = [i32]
             L.jb_status_string.restype = ctypes.c_char_p
             L.jb_debug_philox.argtypes = [jb_seed, u64, u64, vp, vp]
+            L.jb_debug_philox_fold.argtypes = [jb_seed, u64, u64, vp, vp]
             L.jb_debug_gaussian.argtypes = [jb_seed, u64, u64, vp, vp]
             L.jb_debug_box_muller.argtypes = [vp, u64, vp, vp]
             for f in ("jb_perturb", "jb_perturb_with_grid", "jb_apply_updates",
                       "jb_apply_updates_with_grid", "jb_apply_updates_from", "jb_replay_updates",
                       "jb_checksum", "jb_checksum_with_grid", "jb_perturb_q4", "jb_q4_levels",
                       "jb_quantize_grad", "jb_dequantize_grad",
-                      "jb_max_seeds_per_call", "jb_debug_philox", "jb_debug_gaussian",
+                      "jb_max_seeds_per_call", "jb_debug_philox", "jb_debug_philox_fold",
+                      "jb_debug_gaussian",
                       "jb_debug_box_muller"):
                 getattr(L, f).restype = i32
             _lib = L
@@ -321,6 +323,12 @@ def jb_debug_philox(seed, first_block: int, n_blocks: int, out, stream=None) -> 
     """out: CUDA int32/uint32 tensor of >= 4 n_blocks words, 16-byte aligned."""
     _check(lib().jb_debug_philox(_seed(seed), int(first_block), int(n_blocks), out.data_ptr(),
                                  _stream(stream)))
+
+
+def jb_debug_philox_fold(seed, first_block: int, n_blocks: int, out, stream=None) -> None:
+    """out: CUDA int32/uint32 tensor of >= 1 element; receives the XOR of all words."""
+    _check(lib().jb_debug_philox_fold(_seed(seed), int(first_block), int(n_blocks),
+                                      out.data_ptr(), _stream(stream)))
 
 
 def jb_debug_gaussian(seed, first_elem: int, n: int, out, stream=None) -> None:

@@ -1,4 +1,4 @@
-"""Prints the fp32 level and midpoint table of the 4-bit weight code (jb_q4.cuh).
+"""Prints the fp32 level and midpoint table of the 4-bit weight code (jb_q4.cu).
 
     python paper_2306_10015_gb300/csrc/gen_q4_levels.py
 

@@ -123,7 +123,15 @@ double dequantize(int8_t q, double qscale) {
     return q < 0 ? -v : v;
 }
 
-int cuda_status(cudaError_t e) { return e == cudaSuccess ? JB_OK : JB_ERR_CUDA; }
+// libjb links the CUDA runtime statically: its last-error state is its own, so the
+// errors of a caller's runtime (torch's, say) are neither seen nor cleared here. A
+// failed call of this library's is cleared from that state (cudaGetLastError) so that
+// it cannot be reported again by a later, unrelated call.
+int cuda_status(cudaError_t e) {
+    if (e == cudaSuccess) return JB_OK;
+    (void)cudaGetLastError();
+    return JB_ERR_CUDA;
+}
 
 int perturb_impl(const jb_segment* segs, int n_segs, int dtype, jb_seed seed, float eps,
                  int grid_ctas, cudaStream_t stream) {
@@ -518,6 +526,15 @@ JB_EXPORT int jb_debug_philox(jb_seed seed, uint64_t first_block, uint64_t n_blo
     if (reinterpret_cast<uint64_t>(d_out) & 15ull) return JB_ERR_MISALIGNED;  // one 16-byte store per block
     return cuda_status(jb::launch_debug_philox(seed_param(seed, 0.0f), first_block, n_blocks, d_out,
                                                stream));
+}
+
+JB_EXPORT int jb_debug_philox_fold(jb_seed seed, uint64_t first_block, uint64_t n_blocks,
+                                   uint32_t* d_out, struct CUstream_st* stream) {
+    if (d_out == nullptr) return JB_ERR_INVALID_ARG;
+    if (n_blocks > (1ull << 46) || first_block > (1ull << 60)) return JB_ERR_INVALID_ARG;
+    if (reinterpret_cast<uint64_t>(d_out) & 3ull) return JB_ERR_MISALIGNED;
+    return cuda_status(jb::launch_debug_philox_fold(seed_param(seed, 0.0f), first_block, n_blocks,
+                                                    d_out, stream));
 }
 
 JB_EXPORT int jb_debug_gaussian(jb_seed seed, uint64_t first_elem, uint64_t n, float* d_out,

@@ -114,6 +114,8 @@ cudaError_t launch_checksum(const PerturbParams& p, int dtype, unsigned long lon
                             int grid_ctas, cudaStream_t s);
 cudaError_t launch_debug_philox(SeedParam seed, uint64_t first_block, uint64_t n_blocks,
                                 uint32_t* out, cudaStream_t s);
+cudaError_t launch_debug_philox_fold(SeedParam seed, uint64_t first_block, uint64_t n_blocks,
+                                     uint32_t* out, cudaStream_t s);
 cudaError_t launch_debug_gaussian(SeedParam seed, uint64_t first, uint64_t n, float* out,
                                   cudaStream_t s);
 cudaError_t launch_debug_box_muller(const uint32_t* words, uint64_t n_pairs, float* out,

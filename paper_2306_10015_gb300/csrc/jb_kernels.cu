@@ -1,7 +1,8 @@
 // jb_kernels.cu -- sm_103a kernels of the seeded-perturbation hot path.
 //
 //   seeded_kernel<T, false>  PerturbParameters(theta, eps, s) (Algorithm 1,
-//                            subroutine): theta_e <- round_T(fma(eps, z_e, theta_e)).
+//                            subroutine): theta_e <- round_T(theta_e + eps z_e),
+//                            one fused multiply-add fma(s_e, eps r_e, theta_e).
 //   seeded_kernel<T, true>   the step update (Section 2; Algorithm 1):
 //                            theta_e <- round_T(theta_e + sum_k c_k z_e(s_k)),
 //                            the K pairs regenerated in registers, so theta is
@@ -158,6 +159,17 @@ __device__ __forceinline__ void tile_words(const SeedConst& sc, const uint64_t (
                                    static_cast<uint32_t>(blk[j] >> 32));
 }
 
+// acc_even += c z_even, acc_odd += c z_odd for the Gaussians of one Philox block.
+// The scale c is applied to the radius (rc = c r, rounded once) and each product
+// c z is formed as one fused multiply-add of the signed cosine or sine with rc: one
+// packed multiply fewer per block than scaling z = cos r after it is rounded.
+__device__ __forceinline__ void accum_block(uint4 w, float2 c, float2& acc_even, float2& acc_odd) {
+    const Polar2 o = polar2(w);
+    const float2 rc = mul2<kPackO>(c, o.rr);
+    acc_even = fma2<kPackO>(o.cm, rc, acc_even);
+    acc_odd = fma2<kPackO>(o.sm, rc, acc_odd);
+}
+
 // acc += c z for the Gaussians of the words w; accumulators are packed per block as
 // (elements 4b, 4b + 2) and (4b + 1, 4b + 3).
 template <int V, int B>
@@ -166,11 +178,7 @@ __device__ __forceinline__ void tile_accumulate(const uint4 (&w)[V][B], float c,
 #pragma unroll
     for (int j = 0; j < V; ++j)
 #pragma unroll
-        for (int b = 0; b < B; ++b) {
-            const GaussPair g = box_muller2(w[j][b]);
-            acc[j][b][0] = fma2<kPackO>(splat(c), g.even, acc[j][b][0]);
-            acc[j][b][1] = fma2<kPackO>(splat(c), g.odd, acc[j][b][1]);
-        }
+        for (int b = 0; b < B; ++b) accum_block(w[j][b], splat(c), acc[j][b][0], acc[j][b][1]);
 }
 
 template <typename T, bool UPDATE>
@@ -389,11 +397,7 @@ __device__ __forceinline__ void accumulate_range(const P& p, const uint64_t (&bl
                                              static_cast<uint32_t>(blk[j + 1] >> 32));
                 }
 #pragma unroll
-                for (int b = 0; b < B; ++b) {
-                    const GaussPair g = box_muller2(wc[b]);
-                    acc[j][b][0] = fma2<kPackO>(splat(c), g.even, acc[j][b][0]);
-                    acc[j][b][1] = fma2<kPackO>(splat(c), g.odd, acc[j][b][1]);
-                }
+                for (int b = 0; b < B; ++b) accum_block(wc[b], splat(c), acc[j][b][0], acc[j][b][1]);
                 if (j + 1 < V) {
 #pragma unroll
                     for (int b = 0; b < B; ++b) wc[b] = wn[b];
@@ -408,14 +412,19 @@ __device__ __forceinline__ void accumulate_range(const P& p, const uint64_t (&bl
         // and interleave in one instruction stream. The last seed is peeled.
         uint4 w[V][B];
         tile_words<V, B>(seed_const(seed_key(p.seeds[kb])), blk, w);
+        // per block: the next seed's Philox words, then this seed's transform
         for (uint32_t k = kb; k + 1 < ke; ++k) {
-            uint4 wn[V][B];
-            tile_words<V, B>(seed_const(seed_key(p.seeds[k + 1])), blk, wn);
-            tile_accumulate<V, B>(w, p.seeds[k].coef, acc);
+            const SeedConst sn = seed_const(seed_key(p.seeds[k + 1]));
+            const float2 c = splat(p.seeds[k].coef);
 #pragma unroll
             for (int j = 0; j < V; ++j)
 #pragma unroll
-                for (int b = 0; b < B; ++b) w[j][b] = wn[j][b];
+                for (int b = 0; b < B; ++b) {
+                    const uint4 wn = philox_block(sn, static_cast<uint32_t>(blk[j]) + b,
+                                                  static_cast<uint32_t>(blk[j] >> 32));
+                    accum_block(w[j][b], c, acc[j][b][0], acc[j][b][1]);
+                    w[j][b] = wn;
+                }
         }
         tile_accumulate<V, B>(w, p.seeds[ke - 1].coef, acc);
     } else {
@@ -461,14 +470,17 @@ __device__ __forceinline__ void update_tile(const P& p, Tile<T, V>& tl) {
     add_acc<T, V, false>(tl, acc);
 }
 
-// theta <- fma(eps, z, theta) over the tile. The Philox words of vector j + 1 are
-// computed while vector j is transformed, so the integer-multiply and fp32 work
-// of neighbouring vectors interleave (as the update does across seeds).
-template <typename T, int V, typename P>
-__device__ __forceinline__ void perturb_tile(const P& p, Tile<T, V>& tl) {
+// One seed over the tile: ADD = false is the perturbation theta <- fma(., ., theta)
+// (one rounding of theta + eps z); ADD = true is a one-pair update, theta <- theta +
+// (c z rounded to fp32), the same arithmetic as update_tile with K = 1. The Philox
+// words of vector j + 1 are computed while vector j is transformed, so the
+// integer-multiply and fp32 work of neighbouring vectors interleave (as the update
+// does across seeds).
+template <typename T, int V, bool ADD, typename P>
+__device__ __forceinline__ void one_seed_tile(const P& p, Tile<T, V>& tl) {
     constexpr int B = Traits<T>::E / 4;
     const SeedConst sc = seed_const(seed_key(p.seeds[0]));
-    const float2 eps = splat(p.seeds[0].coef);
+    const float2 c = splat(p.seeds[0].coef);
     uint4 wc[B], wn[B];
 #pragma unroll
     for (int b = 0; b < B; ++b)
@@ -483,13 +495,22 @@ __device__ __forceinline__ void perturb_tile(const P& p, Tile<T, V>& tl) {
         }
 #pragma unroll
         for (int b = 0; b < B; ++b) {
-            const GaussPair g = box_muller2(wc[b]);
-            const float2 ev = fma2<kPackO>(eps, g.even, make_float2(tl.x[j][4 * b + 0], tl.x[j][4 * b + 2]));
-            const float2 od = fma2<kPackO>(eps, g.odd, make_float2(tl.x[j][4 * b + 1], tl.x[j][4 * b + 3]));
-            tl.x[j][4 * b + 0] = ev.x;
-            tl.x[j][4 * b + 2] = ev.y;
-            tl.x[j][4 * b + 1] = od.x;
-            tl.x[j][4 * b + 3] = od.y;
+            float* x = &tl.x[j][4 * b];
+            if constexpr (ADD) {
+                float2 ev = make_float2(0.0f, 0.0f), od = make_float2(0.0f, 0.0f);
+                accum_block(wc[b], c, ev, od);
+                x[0] = __fadd_rn(x[0], ev.x);
+                x[2] = __fadd_rn(x[2], ev.y);
+                x[1] = __fadd_rn(x[1], od.x);
+                x[3] = __fadd_rn(x[3], od.y);
+            } else {
+                float2 ev = make_float2(x[0], x[2]), od = make_float2(x[1], x[3]);
+                accum_block(wc[b], c, ev, od);
+                x[0] = ev.x;
+                x[2] = ev.y;
+                x[1] = od.x;
+                x[3] = od.y;
+            }
         }
         if (j + 1 < V) {
 #pragma unroll
@@ -510,7 +531,20 @@ __launch_bounds__(kThreads)
     constexpr int S = UPDATE ? Traits<T>::SU : Traits<T>::SP;
     visit_tiles<T, V, S, false>(p, false, [&](Tile<T, V>& tl) {
         if constexpr (UPDATE) update_tile<T, V>(p, tl);
-        else perturb_tile<T, V>(p, tl);
+        else one_seed_tile<T, V, false>(p, tl);
+    });
+}
+
+// A one-pair update (K = 1, one group) in the perturbation's tile shape: in place
+// (TO_DST = false) or from the source table to the destination (and back to the
+// source when write_src).
+template <typename T, bool TO_DST, typename P>
+__global__ void __launch_bounds__(kThreads) one_pair_kernel(const __grid_constant__ P p) {
+    constexpr int V = Traits<T>::VP;
+    bool also_src = false;
+    if constexpr (TO_DST) also_src = p.write_src != 0;
+    visit_tiles<T, V, Traits<T>::SP, TO_DST>(p, also_src, [&](Tile<T, V>& tl) {
+        one_seed_tile<T, V, true>(p, tl);
     });
 }
 
@@ -678,6 +712,32 @@ __global__ void debug_philox_kernel(SeedParam sp, uint64_t first, uint64_t n, ui
     reinterpret_cast<uint4*>(out)[i] = w;
 }
 
+// The Philox words of blocks [first, first + n) folded by XOR into *out: the
+// generator alone, with the hot path's block function, on a persistent grid (each
+// thread keeps kFoldIlp blocks in flight). XOR is order-free, so the result does
+// not depend on the grid.
+constexpr int kFoldIlp = 4;
+
+__global__ void __launch_bounds__(kThreads) debug_philox_fold_kernel(SeedParam sp, uint64_t first,
+                                                                    uint64_t n, uint32_t* out) {
+    const SeedConst sc = seed_const(seed_key(sp));
+    const uint64_t stride = static_cast<uint64_t>(gridDim.x) * kThreads;
+    uint32_t acc = 0;
+    for (uint64_t i = static_cast<uint64_t>(blockIdx.x) * kThreads + threadIdx.x; i < n;
+         i += kFoldIlp * stride) {
+#pragma unroll
+        for (int u = 0; u < kFoldIlp; ++u) {
+            const uint64_t j = i + u * stride;
+            const uint64_t b = first + j;
+            const uint4 w = philox_block(sc, static_cast<uint32_t>(b), static_cast<uint32_t>(b >> 32));
+            if (j < n) acc ^= w.x ^ w.y ^ w.z ^ w.w;
+        }
+    }
+#pragma unroll
+    for (int d = 16; d > 0; d >>= 1) acc ^= __shfl_xor_sync(0xFFFFFFFFu, acc, d);
+    if ((threadIdx.x & 31u) == 0) atomicXor(out, acc);
+}
+
 __global__ void debug_gaussian_kernel(SeedParam sp, uint64_t first, uint64_t n, float* out) {
     const uint64_t i = static_cast<uint64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
     if (i >= n) return;
@@ -706,7 +766,7 @@ __global__ void debug_box_muller_kernel(const uint32_t* words, uint64_t n, float
 
 // Persistent grid: SM count x resident CTAs per SM, cached per device and kernel.
 constexpr int kMaxDevices = 64;
-constexpr int kKernels = 8;
+constexpr int kKernels = 13;
 std::atomic<int> g_grid_cache[kMaxDevices][kKernels];
 
 template <typename K>
@@ -750,7 +810,29 @@ cudaError_t launch_seeded(const P& p, int slot, int grid_ctas, cudaStream_t stre
 
 }  // namespace
 
+template <typename T, bool TO_DST, typename P>
+cudaError_t launch_one_pair_t(const P& p, int slot, int grid_ctas, cudaStream_t stream) {
+    if (p.n_vec == 0) return cudaSuccess;
+    auto kernel = one_pair_kernel<T, TO_DST, P>;
+    int grid = grid_ctas;
+    if (grid <= 0) {
+        cudaError_t err = persistent_grid(kernel, slot, &grid);
+        if (err != cudaSuccess) return err;
+        constexpr uint64_t vec_per_cta = 32ull * Traits<T>::VP * Traits<T>::SP * (kThreads / 32);
+        const uint64_t needed = (p.n_vec + vec_per_cta - 1) / vec_per_cta;
+        if (needed < static_cast<uint64_t>(grid)) grid = static_cast<int>(needed);
+    }
+    kernel<<<grid, kThreads, 0, stream>>>(p);
+    return cudaGetLastError();
+}
+
 cudaError_t launch_update(const UpdateParams& p, int dtype, int grid_ctas, cudaStream_t s) {
+    // one pair: the perturbation's tile shape (4 vectors per thread, the next
+    // vector's Philox words during the current transform) is faster for one seed
+    if (p.n_seeds == 1) {
+        if (dtype == kF32) return launch_one_pair_t<float, false>(p, 9, grid_ctas, s);
+        return launch_one_pair_t<__nv_bfloat16, false>(p, 10, grid_ctas, s);
+    }
     if (dtype == kF32) return launch_seeded<float, true>(p, 0, grid_ctas, s);
     return launch_seeded<__nv_bfloat16, true>(p, 1, grid_ctas, s);
 }
@@ -772,6 +854,10 @@ cudaError_t launch_general_t(const GeneralParams& p, int slot, int grid_ctas, cu
 }
 
 cudaError_t launch_general(const GeneralParams& p, int dtype, int grid_ctas, cudaStream_t s) {
+    if (p.n_groups == 1 && p.n_seeds == 1) {
+        if (dtype == kF32) return launch_one_pair_t<float, true>(p, 11, grid_ctas, s);
+        return launch_one_pair_t<__nv_bfloat16, true>(p, 12, grid_ctas, s);
+    }
     if (dtype == kF32) return launch_general_t<float>(p, 4, grid_ctas, s);
     return launch_general_t<__nv_bfloat16>(p, 5, grid_ctas, s);
 }
@@ -810,6 +896,19 @@ cudaError_t launch_debug_philox(SeedParam seed, uint64_t first, uint64_t n, uint
                                 cudaStream_t s) {
     if (n == 0) return cudaSuccess;
     debug_philox_kernel<<<blocks_for(n), 256, 0, s>>>(seed, first, n, out);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_debug_philox_fold(SeedParam seed, uint64_t first, uint64_t n, uint32_t* out,
+                                     cudaStream_t s) {
+    cudaError_t err = cudaMemsetAsync(out, 0, sizeof(uint32_t), s);
+    if (err != cudaSuccess || n == 0) return err;
+    int grid = 0;
+    err = persistent_grid(debug_philox_fold_kernel, 8, &grid);
+    if (err != cudaSuccess) return err;
+    const uint64_t needed = (n + kThreads - 1) / kThreads;
+    if (needed < static_cast<uint64_t>(grid)) grid = static_cast<int>(needed);
+    debug_philox_fold_kernel<<<grid, kThreads, 0, s>>>(seed, first, n, out);
     return cudaGetLastError();
 }
 

@@ -6,8 +6,9 @@
 // 64 elements share one fp32 scale, the largest |w| of the block; a weight is
 // level[code] * scale; quantizing picks the nearest level (ties to the lower).
 //
-// Per element: dequantize, w' = fma(eps, z, w) with the same z as every other
-// path (global index flat_offset + i), then per block scale' = max |w'| and
+// Per element: dequantize, w' = w + eps z as one fused multiply-add (as in the
+// plain perturbation) with the same z as every other path (global index
+// flat_offset + i), then per block scale' = max |w'| and
 // code' = nearest level of w' / scale'. Codes and scales are rewritten in place.
 // A 64-element block is four consecutive lanes (16 elements each): its maximum
 // is two butterfly shuffles. Levels live in shared memory, read with
@@ -47,13 +48,16 @@ __constant__ float c_mid[15] = {
 
 // Nearest level of x (ties to the lower): the number of midpoints strictly below
 // x. bucket[j] = (the midpoint in [(j - 16)/16, (j - 15)/16) or +inf, the
-// number of midpoints below (j - 16)/16 as integer bits). x below -1 or NaN
-// takes bucket 0 (code 0, as no midpoint is below it); x at or above 15/16
-// takes bucket 31.
+// number of midpoints below (j - 16)/16 as integer bits). The bucket index
+// floor(16 x) + 16 is read from the fraction bits of x + 3 rounded toward minus
+// infinity: x + 3 lies in [2, 4), where the top five fraction bits are
+// floor(16 (x + 1)), and rounding down never crosses a multiple of 1/16 (all of
+// them are representable there). x is first limited to [-1, 1 - 2^-24]; x below
+// -1 or NaN takes bucket 0 (code 0, as no midpoint is below it).
 __device__ __forceinline__ uint32_t q4_code(float x, const float2* bucket) {
-    const float xc = fmaxf(x, -1.0f);                   // NaN -> -1
-    const int b = min(__float2int_rd(16.0f * xc), 15);  // in [-16, 15]
-    const float2 e = bucket[b + 16];
+    const float xc = fminf(fmaxf(x, -1.0f), 0x1.fffffep-1f);  // NaN -> -1
+    const uint32_t b = (__float_as_uint(__fadd_rd(xc, 3.0f)) >> 18) & 31u;
+    const float2 e = bucket[b];
     return __float_as_uint(e.y) + (x > e.x ? 1u : 0u);
 }
 
@@ -111,11 +115,11 @@ __global__ void __launch_bounds__(kThreadsQ4) q4_perturb_kernel(const __grid_con
         }
         const float sc_in = any ? scale[u >> 2] : 0.0f;
 
-        // dequantize and perturb
-        // the Philox words of block b + 1 are computed while block b is transformed
+        // dequantize and perturb: w = fma(cos or sin, eps r, level * scale), the
+        // Philox words of block b + 1 computed while block b is transformed
         float w[16];
         const uint64_t blk0 = (g.fo + static_cast<uint64_t>(i0)) >> 2;  // fo % 4 == 0
-        float m = 0.0f;
+        const float2 eps2 = splat(eps);
         uint4 wcur = philox_block(sc, static_cast<uint32_t>(blk0), static_cast<uint32_t>(blk0 >> 32));
 #pragma unroll
         for (int b = 0; b < 4; ++b) {
@@ -123,18 +127,31 @@ __global__ void __launch_bounds__(kThreadsQ4) q4_perturb_kernel(const __grid_con
             if (b + 1 < 4)
                 wnext = philox_block(sc, static_cast<uint32_t>(blk0 + b + 1),
                                      static_cast<uint32_t>((blk0 + b + 1) >> 32));
-            const GaussPair z = box_muller2(wcur);
+            const Polar2 o = polar2(wcur);
             if (b + 1 < 4) wcur = wnext;
-            const float zz[4] = {z.even.x, z.odd.x, z.even.y, z.odd.y};
+            const float2 rc = mul2<kPackO>(eps2, o.rr);
+            float lv[4];
 #pragma unroll
             for (int t = 0; t < 4; ++t) {
                 const int k = 4 * b + t;
-                const uint32_t c = (cw[k / 8] >> (4 * (k % 8))) & 0xFu;
-                const float v = __fmaf_rn(eps, zz[t], __fmul_rn(level[c], sc_in));
-                w[k] = v;
-                if (i0 + k < n) m = fmaxf(m, fabsf(v));
+                lv[t] = __fmul_rn(level[(cw[k / 8] >> (4 * (k % 8))) & 0xFu], sc_in);
             }
+            const float2 ev = fma2<kPackO>(o.cm, rc, make_float2(lv[0], lv[2]));
+            const float2 od = fma2<kPackO>(o.sm, rc, make_float2(lv[1], lv[3]));
+            w[4 * b + 0] = ev.x;
+            w[4 * b + 1] = od.x;
+            w[4 * b + 2] = ev.y;
+            w[4 * b + 3] = od.y;
         }
+        // elements past the end of the segment do not count towards the maximum
+        if (!full) {
+#pragma unroll
+            for (int k = 0; k < 16; ++k)
+                if (i0 + k >= n) w[k] = 0.0f;
+        }
+        float m = 0.0f;
+#pragma unroll
+        for (int k = 0; k < 16; ++k) m = fmaxf(m, fabsf(w[k]));
         // block maximum over the four lanes of the block (lanes 4j .. 4j + 3)
         m = fmaxf(m, __shfl_xor_sync(0xFFFFFFFFu, m, 1));
         m = fmaxf(m, __shfl_xor_sync(0xFFFFFFFFu, m, 2));

@@ -82,14 +82,30 @@ __device__ __forceinline__ void philox_round(uint32_t& x0, uint32_t& x1, uint32_
     x2 = y2;
 }
 
-// Four words of Philox4x32-10 block (b_lo, b_hi): round 1 from the per-seed
-// constants, rounds 2 .. 10 in full.
-__device__ __forceinline__ uint4 philox_block(const SeedConst& s, uint32_t b_lo, uint32_t b_hi) {
+// The seed-independent part of round 1 for block (b_lo, b_hi): the product of
+// counter word 0 (the block's low word) and its high word. Every seed of an update
+// shares it.
+struct BlockCtr {
+    uint32_t p_hi, p_lo;  // M0 * b_lo
+    uint32_t b_hi;
+};
+
+__device__ __forceinline__ BlockCtr block_ctr(uint32_t b_lo, uint32_t b_hi) {
     const uint64_t p0 = static_cast<uint64_t>(kPhiloxM0) * b_lo;
-    uint32_t x0 = s.a_hi ^ b_hi ^ s.k0;
+    BlockCtr c;
+    c.p_hi = static_cast<uint32_t>(p0 >> 32);
+    c.p_lo = static_cast<uint32_t>(p0);
+    c.b_hi = b_hi;
+    return c;
+}
+
+// Four words of Philox4x32-10 for block c under the seed's constants: round 1 from
+// the per-seed and per-block products, rounds 2 .. 10 in full.
+__device__ __forceinline__ uint4 philox_block(const SeedConst& s, const BlockCtr& c) {
+    uint32_t x0 = s.a_hi ^ c.b_hi ^ s.k0;
     uint32_t x1 = s.a_lo;
-    uint32_t x2 = static_cast<uint32_t>(p0 >> 32) ^ s.c;
-    uint32_t x3 = static_cast<uint32_t>(p0);
+    uint32_t x2 = c.p_hi ^ s.c;
+    uint32_t x3 = c.p_lo;
     uint32_t k0 = s.k0, k1 = s.k1;
 #pragma unroll
     for (int r = 1; r < 10; ++r) {
@@ -98,6 +114,11 @@ __device__ __forceinline__ uint4 philox_block(const SeedConst& s, uint32_t b_lo,
         philox_round(x0, x1, x2, x3, k0, k1);
     }
     return make_uint4(x0, x1, x2, x3);
+}
+
+// Four words of Philox4x32-10 block (b_lo, b_hi).
+__device__ __forceinline__ uint4 philox_block(const SeedConst& s, uint32_t b_lo, uint32_t b_hi) {
+    return philox_block(s, block_ctr(b_lo, b_hi));
 }
 
 __device__ __forceinline__ float rcp_approx(float x) {
@@ -152,12 +173,13 @@ constexpr bool kPackR = JB_PACK_RADIUS, kPackA = JB_PACK_ANGLE, kPackO = JB_PACK
 // operand (q = 4t/(2+t), L = 2 e ln 2 + 2 ln(1+t) = ln u_a^-2 negated, r0 < 0) and
 // the sign is restored in the final sign masks; round-to-nearest is odd-symmetric,
 // so no rounding differs from the unflipped formulas.
-// even = (z of word pair A's even element, pair B's even element), odd likewise.
-struct GaussPair {
-    float2 even, odd;
+// Polar form: rr = (-r of pair A, -r of pair B); cm, sm = the signed cosines and sines
+// (sign flips of the negated radius included), so z_even = cm rr, z_odd = sm rr.
+struct Polar2 {
+    float2 rr, cm, sm;
 };
 
-__device__ __forceinline__ GaussPair box_muller2(uint4 w) {
+__device__ __forceinline__ Polar2 polar2(uint4 w) {
     // ---- radius ----
     const uint32_t ybA = __float_as_uint(__uint2float_rn((w.x & 0xFFFFFE00u) | 0x100u));
     const uint32_t ybB = __float_as_uint(__uint2float_rn((w.z & 0xFFFFFE00u) | 0x100u));
@@ -174,13 +196,14 @@ __device__ __forceinline__ GaussPair box_muller2(uint4 w) {
     p = fma2<kPackR>(ww, p, splat(kLogR0));
     const float2 lp = fma2<kPackR>(q, mul2<kPackR>(ww, p), q);          // 2 ln(1 + t)
     const float2 fe = make_float2(__int2float_rn(ixA >> 23), __int2float_rn(ixB >> 23));
-    const float2 l_hi = mul2<kPackR>(fe, splat(-kTwoLn2Hi));          // exact
     const float2 l_lo = fma2<kPackR>(fe, splat(-kTwoLn2Lo), lp);
-    const float2 L = add2<kPackR>(l_hi, l_lo);                        // -(-2 ln u_a)
+    // e (2 ln 2)_hi is exact, so L is l_hi + l_lo rounded once
+    const float2 L = fma2<kPackR>(fe, splat(-kTwoLn2Hi), l_lo);         // -(-2 ln u_a)
     const float2 yr = make_float2(rsqrt_approx(-L.x), rsqrt_approx(-L.y));
     const float2 r0 = mul2<kPackR>(L, yr);                            // -r0
-    const float2 m = add2<kPackR>(fma2<kPackR>(r0, r0, l_hi), l_lo);    // r0^2 + L
-    const float2 rr = fma2<kPackR>(m, mul2<kPackR>(splat(0.5f), yr), r0); // -(r0 + corr)
+    const float2 m = fma2<kPackR>(r0, r0, L);                          // r0^2 + L
+    Polar2 o;
+    o.rr = fma2<kPackR>(m, mul2<kPackR>(splat(0.5f), yr), r0); // -(r0 + corr)
 
     // ---- angle ----
     const int32_t waA = static_cast<int32_t>(((w.y << 2) & 0xFFFFFC00u) | 0x200u);
@@ -200,15 +223,25 @@ __device__ __forceinline__ GaussPair box_muller2(uint4 w) {
     // cos < 0 when o1 ^ o2, sin < 0 when o2; one more flip for the negated radius
     const uint32_t tA = w.y ^ (w.y << 1), tB = w.w ^ (w.w << 1);
     const bool swA = (tA & 0x40000000u) != 0u, swB = (tB & 0x40000000u) != 0u;
-    const float2 cm = make_float2(
+    o.cm = make_float2(
         __uint_as_float(__float_as_uint(swA ? S.x : C.x) ^ (tA & 0x80000000u) ^ 0x80000000u),
         __uint_as_float(__float_as_uint(swB ? S.y : C.y) ^ (tB & 0x80000000u) ^ 0x80000000u));
-    const float2 sm = make_float2(
+    o.sm = make_float2(
         __uint_as_float(__float_as_uint(swA ? C.x : S.x) ^ (w.y & 0x80000000u) ^ 0x80000000u),
         __uint_as_float(__float_as_uint(swB ? C.y : S.y) ^ (w.w & 0x80000000u) ^ 0x80000000u));
+    return o;
+}
+
+// even = (z of word pair A's even element, pair B's even element), odd likewise.
+struct GaussPair {
+    float2 even, odd;
+};
+
+__device__ __forceinline__ GaussPair box_muller2(uint4 w) {
+    const Polar2 o = polar2(w);
     GaussPair g;
-    g.even = mul2<kPackO>(cm, rr);
-    g.odd = mul2<kPackO>(sm, rr);
+    g.even = mul2<kPackO>(o.cm, o.rr);
+    g.odd = mul2<kPackO>(o.sm, o.rr);
     return g;
 }
 

@@ -44,7 +44,16 @@ def bf16_ord(h: np.ndarray) -> np.ndarray:
     return np.where(h & 0x8000, -(h & 0x7FFF), h)
 
 
-def check_theta(got: np.ndarray, want: np.ndarray, scale: np.ndarray, what: str = "") -> float:
+# Elements more than one bf16 step from the oracle that the fp32 allowance admits
+# (reading R13: where theta + sum c z cancels, the bf16 steps of the result are finer
+# than the fp32 error of the operands): (what, count, checked) per check_theta call.
+WIDENED = []
+# their largest share of the checked elements in any one call
+BF16_WIDENED_SHARE = 1e-4
+
+
+def check_theta(got: np.ndarray, want: np.ndarray, scale: np.ndarray, what: str = "",
+                max_widened_share: float = BF16_WIDENED_SHARE) -> float:
     """Asserts parity; returns the worst error over its allowance (<= 1 passes)."""
     assert got.shape == want.shape and got.dtype == want.dtype
     if got.dtype == np.uint16:
@@ -59,6 +68,13 @@ def check_theta(got: np.ndarray, want: np.ndarray, scale: np.ndarray, what: str 
         worst = float(r.max()) if r.size else 0.0
         i = int(np.argmax(r)) if r.size else 0
         assert worst <= 1.0, f"{what}: bf16 distance {d[i]} at {i} (|d| {err[i]:.3e}, scale {scale[i]:.3e})"
+        n_wide = int(np.count_nonzero(d > BF16_ULP_TOL))
+        WIDENED.append((what, n_wide, int(d.size)))
+        if n_wide:
+            print(f"{what}: {n_wide} of {d.size} elements beyond one bf16 step, each within "
+                  f"one step + 2e-6 x operands (share {n_wide / d.size:.2e})")
+        assert n_wide <= max_widened_share * d.size + 1, \
+            f"{what}: {n_wide} of {d.size} elements need the widened bf16 allowance"
         return max(worst, float(np.minimum(d, BF16_ULP_TOL).max(initial=0)) / BF16_ULP_TOL)
     d = np.abs(got.astype(np.float64) - want.astype(np.float64))
     allow = F32_REL_TOL * scale + 2.0**-149

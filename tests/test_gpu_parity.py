@@ -16,7 +16,8 @@ import pytest
 
 import oracle
 import synthetic
-from jbtest_util import (Z_ABS_TOL, as_f64, check_theta, to_device, to_host, update_scale)
+from jbtest_util import (WIDENED, Z_ABS_TOL, as_f64, check_theta, to_device, to_host,
+                         update_scale)
 
 torch = pytest.importorskip("torch")
 pytestmark = pytest.mark.gpu
@@ -56,6 +57,19 @@ def test_philox_stream_bit_exact(jb, seed):
         sync()
         got = out.cpu().numpy().view(np.uint32).reshape(n, 4)
         assert np.array_equal(got, oracle.philox_blocks(seed, first, n))
+
+
+@pytest.mark.parametrize("seed", SEEDS[:3])
+def test_philox_fold_bit_exact(jb, seed):
+    """The generator-only kernel (the benchmark's generator floor) folds exactly the
+    words the oracle draws, on ragged counts and across the 2^32-block boundary."""
+    out = torch.zeros(1, dtype=torch.int32, device="cuda")
+    for first, n in ((0, 1 << 20), ((1 << 32) - 5000, 77_777), (7_493_600_000, 1), (12, 0)):
+        jb.jb_debug_philox_fold(seed, first, n, out)
+        sync()
+        got = int(out.cpu().numpy().view(np.uint32)[0])
+        want = int(np.bitwise_xor.reduce(oracle.philox_blocks(seed, first, n).ravel())) if n else 0
+        assert got == want, (first, n)
 
 
 @pytest.fixture(scope="module")
@@ -218,12 +232,12 @@ def test_perturb_parity(jb, dtype, kind):
     seed, eps = (0x1234_5678_9ABC_DEF0, 7, 2), float(F32(1e-3))
     jb.jb_perturb(table, seed, eps)
     sync()
-    worst = 0.0
+    worst, mark = 0.0, len(WIDENED)
     for v, fo, got in zip(vals, offs, download(table)):
         want = oracle.perturb(v, fo, seed, eps)
         z = oracle.gaussian_range(seed, fo, v.size)
         worst = max(worst, check_theta(got, want, np.abs(as_f64(v)) + eps * np.abs(z), kind))
-    print(f"{kind}/{dtype}: worst error / allowance = {worst:.3f}")
+    print(f"{kind}/{dtype}: worst error / allowance = {worst:.3f}; {_widened(mark)}")
 
 
 @pytest.mark.parametrize("dtype", ["f32", "bf16"])
@@ -245,6 +259,13 @@ def test_perturb_restore_cycle(jb, dtype):
         assert np.all(np.abs(as_f64(got) - as_f64(v)) <= 1.5 * ulp + 1e-40)
 
 
+def _widened(mark: int) -> str:
+    """Elements beyond one bf16 step (admitted by the fp32 allowance) since WIDENED[mark]."""
+    n = sum(w for _, w, _ in WIDENED[mark:])
+    tot = sum(t for _, _, t in WIDENED[mark:])
+    return f"{n} of {tot} elements beyond one bf16 step" if tot else "fp32"
+
+
 def _pairs(K, step=3, stream=0):
     mids = synthetic.machine_ids(K, 20 + stream)
     seeds = [(int(m), step, int(i % 3)) for i, m in enumerate(mids)]
@@ -261,13 +282,13 @@ def test_update_parity(jb, dtype, K, kind):
     seeds, q = _pairs(K)
     jb.jb_apply_updates(table, seeds, q, LR, DENOM, QS)
     sync()
-    worst = 0.0
+    worst, mark = 0.0, len(WIDENED)
     for v, fo, got in zip(vals, offs, download(table)):
         want = oracle.update(v, fo, seeds, q, LR, DENOM, QS)
         idx = np.arange(fo, fo + v.size, dtype=np.uint64)
         scale = update_scale(v, idx, seeds, q, LR, DENOM, QS)
         worst = max(worst, check_theta(got, want, scale, f"{kind} K={K}"))
-    print(f"{kind}/{dtype}/K={K}: worst error / allowance = {worst:.3f}")
+    print(f"{kind}/{dtype}/K={K}: worst error / allowance = {worst:.3f}; {_widened(mark)}")
 
 
 def test_update_k256_parity(jb):

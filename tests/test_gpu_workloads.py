@@ -14,7 +14,8 @@ import pytest
 
 import oracle
 import synthetic
-from jbtest_util import as_f64, bf16_ord, check_theta, to_device, to_host, update_scale
+from jbtest_util import (WIDENED, as_f64, bf16_ord, check_theta, to_device, to_host,
+                         update_scale)
 
 torch = pytest.importorskip("torch")
 pytestmark = pytest.mark.gpu
@@ -156,34 +157,50 @@ def test_toy_spsa_run_matches_oracle(jb):
 
 
 def test_dynamic_membership_30b(jb):
-    """OPT-30B-shaped bf16 (772 tensors, ~60 GB): 20 steps, 1..512 machines per
-    step drawn from a pool of 1024 non-contiguous ids, denom = K_t; the final
-    theta checked on sampled indices against the oracle run from the same start."""
-    table, pos, offs = _setup(jb, "opt-30b", "bf16", n_samples=1 << 17)
+    """OPT-30B-shaped bf16 (772 tensors, ~60 GB): 20 steps, 1..512 machines per step
+    drawn from a pool of 1024 non-contiguous ids, denom = K_t; 2^22 sampled indices
+    checked in two modes (Algorithm 1's gradient loop; Section 2, machines joining
+    and leaving):
+      stepwise      each step's oracle input is the GPU's theta at that step's start;
+                    every sampled element is within one bf16 step of the oracle (R13:
+                    beyond it only where the fp32 allowance of the operands admits it,
+                    for at most BF16_WIDENED_SHARE of the elements of a step);
+      free-running  the oracle runs all 20 steps from the same start; the bf16-step
+                    histogram is printed and every element lies within the allowance
+                    accumulated over the steps."""
+    n_samples = 1 << 22
+    table, pos, offs = _setup(jb, "opt-30b", "bf16", n_samples=n_samples)
     idx = global_index(offs, pos)
-    vals = gather(table.tensors, pos)
-    start = vals.copy()
+    before = gather(table.tensors, pos)
+    start, free = before.copy(), before.copy()
     lr, qs = float(F32(1e-4)), 16.0
-    Ks = []
+    Ks, wide = [], 0
     allowance = np.zeros(idx.size)
     for t, active in enumerate(synthetic.membership_schedule(20)):
         seeds = [(int(m), t, 0) for m in active]
         q = synthetic.byte_codes(len(seeds), 700 + t)
-        Ks.append(len(seeds))
-        jb.jb_apply_updates(table, seeds, q, lr, float(len(seeds)), qs)
-        # each step may add one bf16 step of its operands plus the fp32 allowance
-        scale = update_scale(vals, idx, seeds, q, lr, float(len(seeds)), qs)
+        K = len(seeds)
+        Ks.append(K)
+        jb.jb_apply_updates(table, seeds, q, lr, float(K), qs)
+        after = gather(table.tensors, pos)
+        # one oracle evaluation of sum c z and sum |c z| serves both modes
+        delta, mag = oracle.update_delta_abs_at(idx, seeds, q, lr, float(K), qs)
+        mark = len(WIDENED)
+        check_theta(after, oracle.round_bf16(as_f64(before) + delta), np.abs(as_f64(before)) + mag,
+                    f"30B stepwise t={t} K={K}")
+        wide += WIDENED[mark][1]
+        scale = np.abs(as_f64(free)) + mag
         allowance += np.ldexp(1.0, np.frexp(scale)[1] - 8) + 2e-6 * scale
-        vals = oracle.update_at(vals, idx, seeds, q, lr, float(len(seeds)), qs)
-    torch.cuda.synchronize()
-    got = gather(table.tensors, pos)
-    d = np.abs(bf16_ord(got) - bf16_ord(vals))
+        free = oracle.round_bf16(as_f64(free) + delta)
+        before = after
+    d = np.abs(bf16_ord(before) - bf16_ord(free))
     hist = np.bincount(np.minimum(d, 64).astype(np.int64))
-    err = np.abs(as_f64(got) - as_f64(vals))
-    print(f"K_t = {Ks}; sampled {idx.size}; bf16 step histogram {hist.tolist()}; "
-          f"worst error / allowance {float((err / allowance).max()):.3f}")
+    err = np.abs(as_f64(before) - as_f64(free))
+    print(f"K_t = {Ks}; sampled {idx.size} of {sum(t.numel() for t in table.tensors)} "
+          f"({idx.size / sum(t.numel() for t in table.tensors):.2e}); stepwise: {wide} element-steps "
+          f"beyond one bf16 step of {idx.size * len(Ks)}; free-running bf16 step histogram "
+          f"{hist.tolist()}; worst error / allowance {float((err / allowance).max()):.3f}")
     assert np.all(err <= allowance)
-    assert hist[0] >= 0.99 * d.size
-    assert not np.array_equal(got, start)
+    assert not np.array_equal(before, start)
     del table
     free_cuda()
