@@ -349,7 +349,8 @@ def main():
         "gpu_launches": launches_per_step * a.steps, "clocks": clk,
     }
     if sweep_lines:
-        out["sweep"] = [roof.report(ln["K"], ln["ms"]) if "K" in ln else ln for ln in sweep_lines]
+        out["sweep"] = [roof.report(ln["K"], ln["ms"]) if "K" in ln and "leg" not in ln else ln
+                        for ln in sweep_lines]
     print(json.dumps(out), flush=True)
     if dist is not None:
         dist.destroy_process_group()
