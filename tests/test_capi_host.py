@@ -234,3 +234,13 @@ def test_debug_hooks_check_alignment(jb):
     assert L.jb_debug_box_muller(ctypes.c_void_p(FAKE), 4, ctypes.c_void_p(FAKE + 2), None) == -3
     assert L.jb_debug_gaussian(seed, 0, (1 << 38) + 1, ctypes.c_void_p(FAKE), None) == -1
     assert L.jb_debug_gaussian(seed, 0, 4, None, None) == -1
+
+
+def test_philox_fold_validation(jb):
+    """The generator-only hook refuses a missing, misaligned or oversized request
+    before anything is enqueued."""
+    L, seed = jb.lib(), jb.jb_seed(1, 2, 3)
+    assert L.jb_debug_philox_fold(seed, 0, 4, None, None) == -1
+    assert L.jb_debug_philox_fold(seed, 0, 4, ctypes.c_void_p(FAKE + 2), None) == -3
+    assert L.jb_debug_philox_fold(seed, 0, (1 << 46) + 1, ctypes.c_void_p(FAKE), None) == -1
+    assert L.jb_debug_philox_fold(seed, (1 << 60) + 1, 4, ctypes.c_void_p(FAKE), None) == -1

@@ -274,8 +274,8 @@ def _pairs(K, step=3, stream=0):
 
 
 @pytest.mark.parametrize("dtype", ["f32", "bf16"])
-@pytest.mark.parametrize("K", [1, 3, 17, 64])
-@pytest.mark.parametrize("kind", ["ragged", "phase", "high"])
+@pytest.mark.parametrize("K", [1, 2, 3, 17, 64])
+@pytest.mark.parametrize("kind", ["ragged", "phase", "high", "tiny"])
 def test_update_parity(jb, dtype, K, kind):
     vals, offs, shifts = make_layout(kind, dtype)
     table = upload(jb, vals, offs, shifts)
@@ -302,6 +302,24 @@ def test_update_k256_parity(jb):
         want = oracle.update(v, fo, seeds, q, LR, 256.0, QS)
         idx = np.arange(fo, fo + v.size, dtype=np.uint64)
         check_theta(got, want, update_scale(v, idx, seeds, q, LR, 256.0, QS), "K=256")
+
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_update_max_pairs_parity(jb, dtype):
+    """K = jb_max_seeds_per_call() (512): the largest list one launch carries."""
+    K = jb.jb_max_seeds_per_call()
+    vals, offs, shifts = make_layout("phase", dtype)
+    vals, offs, shifts = vals[:5], offs[:5], shifts[:5]
+    table = upload(jb, vals, offs, shifts)
+    seeds, q = _pairs(K, stream=6)
+    jb.jb_apply_updates(table, seeds, q, LR, float(F32(K)), QS)
+    sync()
+    mark = len(WIDENED)
+    for v, fo, got in zip(vals, offs, download(table)):
+        want = oracle.update(v, fo, seeds, q, LR, float(K), QS)
+        idx = np.arange(fo, fo + v.size, dtype=np.uint64)
+        check_theta(got, want, update_scale(v, idx, seeds, q, LR, float(K), QS), f"K={K}")
+    print(f"K={K}/{dtype}: {_widened(mark)}")
 
 
 @pytest.mark.parametrize("dtype", ["f32", "bf16"])
@@ -341,11 +359,13 @@ def test_repeatable_across_runs_grids_and_splits(jb, dtype):
     v = synthetic.normal_values(n, 0.02, 90)
     v = v if dtype == "f32" else oracle.round_bf16(v.astype(np.float64))
     seeds, q = _pairs(9)
+    one_s, one_q = _pairs(1, stream=4)  # K = 1 takes the one-pair kernel
     ref = None
     for grid in (0, 0, 1, 7, 152, 1000):
         t = upload(jb, [v], [fo], [0])
         jb.jb_apply_updates(t, seeds, q, LR, DENOM, QS, grid_ctas=grid)
         jb.jb_perturb(t, seeds[0], 1e-3, grid_ctas=grid)
+        jb.jb_apply_updates(t, one_s, one_q, LR, DENOM, QS, grid_ctas=grid)
         sync()
         out = download(t)[0]
         if ref is None:
@@ -356,6 +376,7 @@ def test_repeatable_across_runs_grids_and_splits(jb, dtype):
     t = upload(jb, parts, [fo + a for a in cuts[:-1]], [(i * 5) % 8 for i in range(len(parts))])
     jb.jb_apply_updates(t, seeds, q, LR, DENOM, QS)
     jb.jb_perturb(t, seeds[0], 1e-3)
+    jb.jb_apply_updates(t, one_s, one_q, LR, DENOM, QS)
     sync()
     assert np.array_equal(np.concatenate(download(t)), ref)
 
