@@ -57,7 +57,7 @@ def parse():
     ap.add_argument("--lr", type=float, default=1e-6)
     ap.add_argument("--qscale", type=float, default=16.0)
     ap.add_argument("--e2e-steps", type=int, default=4)
-    ap.add_argument("--e2e-groups", type=int, default=32, help="tensor groups of the e2e pipeline")
+    ap.add_argument("--e2e-groups", type=int, default=16, help="tensor groups of the e2e pipeline")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=10.0,

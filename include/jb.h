@@ -13,8 +13,8 @@
  *   jb_apply_updates  the step update: every machine's (seed, one-byte
  *                     projected gradient) pair applied with weight
  *                     -grad * eta / numel(all_grads) in machine-timestamp
- *                     order (Section 2, "Applying collected scalar projected
- *                     gradients"; Algorithm 1), fused into one read and one
+ *                     order (Section 2, on applying the collected scalar projected
+ *                     gradients; Algorithm 1), fused into one read and one
  *                     write of theta.
  *   jb_quantize_grad  the one-byte projected gradient: the logarithm of its
  *   jb_dequantize_grad magnitude with its sign, limited to +-127 (Section 3,

@@ -223,8 +223,8 @@ float jbo_coefficient(int8_t q, double lr, double denom, double qscale) {
 }
 
 /* ------------------------------------------------------------------------ */
-/* Applying collected projected gradients in machine-timestamp order          */
-/* (Section 2; Algorithm 1).                                                  */
+/* The step update: every machine's projected gradients, taken in the order  */
+/* of the machines' start times (Section 2; Algorithm 1).                     */
 /* ------------------------------------------------------------------------ */
 static int seed_cmp(const jbo_seed* a, const jbo_seed* b) {
     if (a->machine_id != b->machine_id) return a->machine_id < b->machine_id ? -1 : 1;

@@ -20,7 +20,9 @@
 //   angle   the 24-bit angle index splits into an octant (3 bits, handled
 //           exactly by reflection, swap and sign flips) and a 21-bit offset
 //           x in (0, 1) of the octant, sin(pi x / 4) and cos(pi x / 4) by
-//           minimax polynomials (relative error < 0.6 ulp, also near zero).
+//           minimax polynomials of degree 7 and 6 (relative error < 0.6 ulp
+//           for the sine, also near zero; 1.0e-7 for the cosine, which the
+//           octant keeps above 0.7).
 // Coefficients: fit_poly.py (Remez exchange). The transform is checked
 // against a double-precision evaluation of the same definition over all
 // radius words and all angle words (|dz| <= 1e-6).
@@ -40,8 +42,7 @@ constexpr float kLogR0 = 0x1.5555b4p-6f, kLogR1 = 0x1.992aaap-11f, kLogR2 = 0x1.
 constexpr float kSinHi = 0x1.921fb6p-1f;   // pi/4 = hi + lo
 constexpr float kSinLo = -0x1.777a5cp-26f;
 constexpr float kSinS0 = -0x1.4abbbep-4f, kSinS1 = 0x1.465facp-9f, kSinS2 = -0x1.2db5cep-15f;
-constexpr float kCosC0 = -0x1.3bd3ccp-2f, kCosC1 = 0x1.03c1b0p-6f, kCosC2 = -0x1.55b2b6p-12f,
-                kCosC3 = 0x1.d4f7eep-19f;
+constexpr float kCosC0 = -0x1.3bd39cp-2f, kCosC1 = 0x1.03b058p-6f, kCosC2 = -0x1.4e78bep-12f;
 constexpr float kTwoLn2Hi = -0x1.62e4p+0f;       // -(2 ln 2) to 16 bits
 constexpr float kTwoLn2Lo = -0x1.7f7d1cp-19f;    // -(2 ln 2) - kTwoLn2Hi
 
@@ -215,8 +216,7 @@ __device__ __forceinline__ Polar2 polar2(uint4 w) {
     ps = fma2<kPackA>(y, ps, splat(kSinS0));
     ps = fma2<kPackA>(y, ps, splat(kSinLo));
     const float2 S = fma2<kPackA>(x, splat(kSinHi), mul2<kPackA>(x, ps));
-    float2 pc = fma2<kPackA>(y, splat(kCosC3), splat(kCosC2));
-    pc = fma2<kPackA>(y, pc, splat(kCosC1));
+    float2 pc = fma2<kPackA>(y, splat(kCosC2), splat(kCosC1));
     pc = fma2<kPackA>(y, pc, splat(kCosC0));
     const float2 C = fma2<kPackA>(y, pc, splat(1.0f));
     // octant bits o2 o1 o0 = word bits 31..29: |cos| and |sin| swap when o0 ^ o1;

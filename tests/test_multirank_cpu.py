@@ -4,7 +4,7 @@
 * The method's data-parallel exchange (Section 2; Algorithm 1): each rank is a
   machine; it evaluates its own SPSA sample on the toy quadratic with the
   oracle, quantizes it to one byte, the (seed, byte) pairs are all-gathered
-  (standing in for the paper's network call), and every rank applies the full
+  (standing in for the method's exchange step), and every rank applies the full
   list. The replicas must stay bitwise identical (checksum and bytes).
 """
 import os
