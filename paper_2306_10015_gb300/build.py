@@ -21,7 +21,7 @@ LIB = os.path.join(OUT_DIR, "libjb.so")
 
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 SOURCES = ["jb_kernels.cu", "jb_q4.cu", "jb_capi.cpp"]
-HEADERS = ["jb_rng.cuh", "jb_internal.h"]
+HEADERS = ["jb_rng.cuh", "jb_internal.h", "jb_q4.h"]
 
 
 def nvcc() -> str:

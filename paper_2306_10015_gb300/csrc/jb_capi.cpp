@@ -14,6 +14,7 @@
 
 #include "jb.h"
 #include "jb_internal.h"
+#include "jb_q4.h"
 
 #define JB_EXPORT extern "C" __attribute__((visibility("default")))
 
@@ -460,7 +461,7 @@ int perturb_q4_impl(const jb_q4_segment* segs, int n_segs, jb_seed seed, float e
             g.fo = q.fo;
             g.n = q.n;
             g.unit0 = unit;
-            unit += 4 * ((q.n + 63) / 64);  // whole 64-element blocks of 16-element units
+            unit += jb::kQ4UnitsPerBlock * ((q.n + 63) / 64);  // whole 64-element blocks
         }
         params.n_segs = static_cast<uint32_t>(count);
         params.n_units = unit;
