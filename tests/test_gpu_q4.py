@@ -26,7 +26,7 @@ def jb():
     return pkg
 
 
-SIZES = [1, 2, 63, 64, 65, 127, 1000, 4097, 64 * 300 + 33]
+SIZES = [1, 2, 31, 32, 33, 63, 64, 65, 96, 97, 127, 1000, 4097, 64 * 300 + 33]
 
 
 def make(jb, sizes, offs, stream=70):
