@@ -444,26 +444,20 @@ class Roofline:
 class E2EPipeline:
     """Theta in pinned host memory, one step at a time through the public calls.
 
-    The tensors are split into n_groups groups of consecutive tensors of about
-    equal bytes. Each group lives in one pinned host buffer and one device buffer,
-    and its tensors are views into them (64-element aligned), so a group moves in
-    one copy each way. Three streams pipeline the groups: group g + 1 arrives while
-    group g is transformed, and group g - 1 leaves. z depends only on the global
-    index, so any split of the table gives the same bits."""
+    The tensors are split into n_groups groups. Each group lives in one pinned host
+    buffer and one device buffer, and its tensors are views into them (64-element
+    aligned), so a group moves in one copy each way. Three streams pipeline the
+    groups: group g + 1 arrives while group g is transformed, and group g - 1
+    leaves. Only the first group's copy in and the last group's copy out are not
+    hidden behind compute, so the groups ramp up and down geometrically (1/16, 1/8,
+    1/4, 1/2 of a middle group at each end) and the smallest tensors are placed at
+    the two ends to make those groups small. z depends only on the global index,
+    so any order and split of the table gives the same bits."""
 
     def __init__(self, jb, tensors, offs, stream, n_groups=32):
         import torch
         self.jb, self.stream = jb, stream
-        total = sum(t.numel() for t in tensors)
-        groups, cur, acc = [], [], 0
-        for i, t in enumerate(tensors):
-            cur.append(i)
-            acc += t.numel()
-            if acc >= total * (len(groups) + 1) / n_groups and len(groups) < n_groups - 1:
-                groups.append(cur)
-                cur = []
-        if cur:
-            groups.append(cur)
+        groups = self.split(tensors, n_groups)
         pad = lambda n: -(-n // 64) * 64
         self.dev_bufs, self.host_bufs = [], []
         self.views, self.host_views = [None] * len(tensors), [None] * len(tensors)
@@ -487,6 +481,46 @@ class E2EPipeline:
         self.tables = [jb.ParamTable([self.views[i] for i in g], [offs[i] for i in g]) for g in groups]
         self.s_in, self.s_out = torch.cuda.Stream(), torch.cuda.Stream()
         self.out_done = [None] * len(groups)
+
+    @staticmethod
+    def split(tensors, n_groups):
+        """Groups of tensor indices: the smallest tensors at both ends of the order,
+        group sizes ramping geometrically at both ends, every group non-empty."""
+        sizes = [t.numel() for t in tensors]
+        n = len(sizes)
+        n_groups = max(1, min(n_groups, n))
+        ramp = min(4, (n_groups - 1) // 2)
+        w = [1.0] * n_groups
+        for i in range(ramp):
+            w[i] = w[n_groups - 1 - i] = 2.0 ** (i - ramp)
+        # order: small tensors alternately to the front and the back, the rest between
+        by_size = sorted(range(n), key=lambda i: sizes[i])
+        total = sum(sizes)
+        end_budget = total * sum(w[:ramp]) / sum(w)
+        front, back, used, acc = [], [], set(), 0
+        for k, i in enumerate(by_size):
+            if acc >= 2 * end_budget:
+                break
+            (front if k % 2 == 0 else back).append(i)
+            used.add(i)
+            acc += sizes[i]
+        order = front + [i for i in range(n) if i not in used] + back[::-1]
+        bounds, c = [], 0.0
+        for x in w[:-1]:
+            c += x
+            bounds.append(total * c / sum(w))
+        groups, cur, acc = [], [], 0
+        for k, i in enumerate(order):
+            cur.append(i)
+            acc += sizes[i]
+            left = n - 1 - k  # tensors not yet placed
+            need = n_groups - 1 - len(groups)  # groups still to open after this one
+            if len(groups) < n_groups - 1 and (acc >= bounds[len(groups)] or left == need):
+                groups.append(cur)
+                cur = []
+        if cur:
+            groups.append(cur)
+        return groups
 
     def step(self, s_own, seeds, q, eps, lr, qscale):
         """Enqueue one step: per group copy in, perturb +eps/-2 eps/+eps, update, copy out."""
