@@ -67,8 +67,12 @@ def parse():
     ap.add_argument("--no-sweep", action="store_true", help="skip the K sweep")
     ap.add_argument("--sweep-out", default="", help="file for the sweep's JSON lines")
     ap.add_argument("--next-legs", action="store_true",
-                    help="with --sweep: also time the backup-fused update and the replay")
-    return ap.parse_args()
+                    help="(the default) with the sweep, also time the backup-fused update, the "
+                         "replay, the checksum and the 4-bit perturbation")
+    ap.add_argument("--no-next-legs", action="store_true", help="skip those legs")
+    a = ap.parse_args()
+    a.next_legs = not a.no_next_legs
+    return a
 
 
 def aggregate_ranks(ms_local: float, units_local: float, dist=None, device=None):
@@ -314,9 +318,9 @@ def main():
         e2e = run_e2e(a, jb, tensors, offs, seeds, codes, ghat, mids, own, stream, N, esize,
                       units_per_step, dist, a.e2e_groups)
 
-    sweep_lines = []
+    sweep_lines, next_lines = [], []
     if a.sweep and not a.no_sweep and rank == 0:
-        sweep_lines = run_sweep(a, jb, table, mids, stream)
+        sweep_lines, next_lines = run_sweep(a, jb, table, mids, stream)
 
     if rank != 0:
         if dist is not None:
@@ -350,8 +354,9 @@ def main():
         "gpu_launches": launches_per_step * a.steps, "clocks": clk,
     }
     if sweep_lines:
-        out["sweep"] = [roof.report(ln["K"], ln["ms"]) if "K" in ln and "leg" not in ln else ln
-                        for ln in sweep_lines]
+        out["sweep"] = [roof.report(ln["K"], ln["ms"]) if "K" in ln else ln for ln in sweep_lines]
+    if next_lines:
+        out["next"] = [roof.leg(ln) for ln in next_lines]
     print(json.dumps(out), flush=True)
     if dist is not None:
         dist.destroy_process_group()
@@ -410,6 +415,24 @@ class Roofline:
         self.N, self.esize, self.gen_rate = N, esize, gen_rate
         self.lanes = self.sms * LANES_PER_SM_CLK * self.f_max
         self.instr = load_instr_per_param_seed(a)
+
+    def leg(self, ln):
+        """A NEXT-row leg with its roofline: the backup-fused update and the replay
+        against the update's (the same bytes per pass and work per element-seed;
+        the backup refresh adds one write), the checksum and the 4-bit pass against
+        the measured copy bandwidth."""
+        ln = dict(ln)
+        if ln.get("mode") in ("fused", "fused+refresh", "replay"):  # one pass over theta
+            k = ln["K"] if ln["leg"] == "restore+update" else ln["steps"] * ln["K_per_step"]
+            t = ln["ms"] / 1e3
+            extra = 1.5 if ln.get("mode") == "fused+refresh" else 1.0
+            t_hbm = extra * 2 * self.esize * self.N / (self.hbm_peak * 1e9)
+            t_alg = OPS_PER_PARAM_SEED * k * self.N / self.lanes
+            ln["frac"] = max(t_hbm, t_alg) / t
+            ln["generator_floor"] = k * self.N / self.gen_rate / t
+        elif ln.get("leg") in ("checksum", "perturb_q4"):
+            ln["hbm_frac"] = ln["hbm_gbs"] / self.hbm_peak
+        return ln
 
     def report(self, K, ms_list):
         st = stats(ms_list)
@@ -667,15 +690,16 @@ def run_sweep(a, jb, table, mids, stream):
     out.append({"perturb_ms": st["mean"], "perturb_ms_best": st["best"], "perturb_ms_median": st["median"],
                 "param_seed_per_s": N / (st["best"] / 1e3),
                 "hbm_gbs": 2 * es * N / (st["best"] / 1e3) / 1e9})
+    nxt = []
     if a.next_legs:
-        out.extend(next_legs(a, jb, table, stream))
-        out.append(checksum_leg(jb, table, stream))
-        out.append(q4_leg(a, jb, stream))
+        nxt.extend(next_legs(a, jb, table, stream))
+        nxt.append(checksum_leg(jb, table, stream))
+        nxt.append(q4_leg(a, jb, stream))
     if a.sweep_out:
         with open(a.sweep_out, "w") as f:
-            for ln in out:
+            for ln in out + nxt:
                 f.write(json.dumps(ln) + "\n")
-    return out
+    return out, nxt
 
 
 def next_legs(a, jb, table, stream):
