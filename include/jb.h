@@ -200,8 +200,14 @@ typedef struct {
  * w'_i = w_i + eps z_i(seed) in fp32, one fused multiply-add as in jb_perturb, then
  * scale' = max_i |w'_i| and code'_i = the nearest level to w'_i / scale' (ties
  * to the lower level; scale' = 0 gives the zero level). Codes and scales are
- * rewritten in place, asynchronously on `stream`. The paper fixes no 4-bit
+ * rewritten in place, asynchronously on `stream`; an odd numel leaves the
+ * unused high nibble of the last byte as it was. The paper fixes no 4-bit
  * format; this is a NormalFloat-style code after QLoRA (see jb_q4_levels).
+ * Errors, found before anything is enqueued: JB_ERR_INVALID_ARG for n_segs < 0,
+ * a null array or pointer, a non-finite eps, an index range past 2^62, or
+ * tensors whose bytes or index ranges overlap; JB_ERR_MISALIGNED for codes not
+ * 8-byte aligned, scale not 4-byte aligned or flat_offset not a multiple of 4.
+ * Tensors with numel = 0 are skipped.
  */
 int jb_perturb_q4(const jb_q4_segment* segs, int n_segs, jb_seed seed, float eps,
                   struct CUstream_st* stream);

@@ -223,6 +223,18 @@ def test_q4_levels_match_oracle_and_validation(jb):
     assert L.jb_perturb_q4(seg, 1, jb.jb_seed(1, 0, 0), 1e-3, None) == -1
     seg[0] = jb.jb_q4_segment(0, FAKE, 100, 8)
     assert L.jb_perturb_q4(seg, 1, jb.jb_seed(1, 0, 0), 1e-3, None) == -1
+    seg[0] = jb.jb_q4_segment(FAKE, FAKE + 4098, 100, 8)           # scale not 4-byte aligned
+    assert L.jb_perturb_q4(seg, 1, jb.jb_seed(1, 0, 0), 1e-3, None) == -3
+    seg[0] = jb.jb_q4_segment(FAKE, FAKE + 4096, 100, (1 << 62) - 96)  # index range past 2^62
+    assert L.jb_perturb_q4(seg, 1, jb.jb_seed(1, 0, 0), 1e-3, None) == -1
+    assert L.jb_perturb_q4(seg, -1, jb.jb_seed(1, 0, 0), 1e-3, None) == -1
+    two = (jb.jb_q4_segment * 2)()
+    two[0] = jb.jb_q4_segment(FAKE, FAKE + 4096, 100, 8)
+    two[1] = jb.jb_q4_segment(FAKE + 8192, FAKE + 12288, 100, 104)  # index ranges overlap
+    assert L.jb_perturb_q4(two, 2, jb.jb_seed(1, 0, 0), 1e-3, None) == -1
+    two[0] = jb.jb_q4_segment(FAKE + 4, FAKE + 2, 0, 6)             # empty tensors are skipped,
+    two[1] = jb.jb_q4_segment(0, 0, 0, 0)                           # unchecked: nothing to launch
+    assert L.jb_perturb_q4(two, 2, jb.jb_seed(1, 0, 0), 1e-3, None) == 0
 
 
 def test_debug_hooks_check_alignment(jb):
