@@ -172,3 +172,60 @@ def test_q4_perturb_large_sampled(jb):
             ok = _check_codes(got, codes_of(oc, m), w, os_, eps, mids)
             n_bad += int(np.sum(~ok))
     assert n_bad == 0
+
+
+def test_q4_perturb_full_size_13b_sampled(jb):
+    """The OPT-13B-shaped set stored as 4-bit codes (12,853,473,280 elements in 644
+    tensors, 6.4 GB of codes), perturbed in the launch the benchmark times; 4096
+    random 64-element blocks, drawn over the whole set, each recomputed by the
+    oracle from its codes and scale before the pass."""
+    specs = synthetic.opt_tensors("opt-13b")
+    g = torch.Generator(device="cuda")
+    g.manual_seed(synthetic.MASTER_SEED + 41)
+    tensors = []
+    for sp in specs:
+        n = sp.numel
+        codes = torch.randint(0, 256, ((n + 1) // 2 + 8,), dtype=torch.uint8, device="cuda", generator=g)
+        scale = torch.rand(((n + 63) // 64,), device="cuda", generator=g) * 0.05
+        tensors.append((codes, scale, n))
+    table = jb.Q4Table(tensors)
+    n_blocks = np.array([(n + 63) // 64 for _, _, n in tensors], dtype=np.int64)
+    first = np.concatenate([[0], np.cumsum(n_blocks)])
+    pick = synthetic.rng(97).choice(int(first[-1]), size=4096, replace=False)
+    which = np.searchsorted(first, pick, side="right") - 1
+    ar = torch.arange(32, device="cuda")
+
+    def gather():
+        out = {}
+        for t in np.unique(which):
+            codes, scale, n = tensors[t]
+            bl = torch.from_numpy(pick[which == t] - first[t]).cuda()
+            idx = (32 * bl[:, None] + ar[None, :]).clamp_(max=codes.numel() - 1)
+            out[int(t)] = (bl.cpu().numpy(), codes[idx].cpu().numpy(), scale[bl].cpu().numpy())
+        return out
+
+    before = gather()
+    seed = (0x5EED_0013_B000, 11, 2)
+    eps = float(F32(1e-3))
+    jb.jb_perturb_q4(table, seed, eps)
+    torch.cuda.synchronize()
+    after = gather()
+    lev = oracle.q4_levels().astype(np.float64)
+    mids = (lev[:-1] + lev[1:]) / 2
+    n_bad = n_checked = 0
+    for t, (bl, c0, s0) in before.items():
+        _, c1, s1 = after[t]
+        n = tensors[t][2]
+        fo = table.flat_offsets[t]
+        for k, b in enumerate(bl):
+            m = int(min(64, n - 64 * b))
+            nb = (m + 1) // 2
+            oc, os_, w = oracle.q4_perturb(c0[k, :nb].copy(), s0[k:k + 1], m, fo + 64 * int(b), seed, eps)
+            assert abs(float(s1[k]) - float(os_[0])) <= 2e-6 * float(os_[0]) + 2e-6 * eps, (t, b)
+            ok = _check_codes(codes_of(c1[k, :nb], m), codes_of(oc, m), w, os_, eps, mids)
+            n_bad += int(np.sum(~ok))
+            n_checked += m
+    print(f"13B-shaped 4-bit set: {n_checked} elements in {len(pick)} blocks checked")
+    assert n_bad == 0
+    del tensors, table
+    torch.cuda.empty_cache()
