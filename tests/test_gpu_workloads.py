@@ -98,6 +98,59 @@ def test_full_size_update_sampled(jb, model, dtype, K):
     free_cuda()
 
 
+@pytest.mark.parametrize("K,write_src", [(1, False), (4, True)])
+def test_full_size_apply_from_sampled_13b(jb, K, write_src):
+    """The update read from the weight backup (Algorithm 1's restore fused) on the
+    13B-shaped bf16 set, in the launches the benchmark times: K = 1 runs the
+    one-pair kernel, K = 4 the grouped kernel with the backup refreshed."""
+    backup, pos, offs = _setup(jb, "opt-13b", "bf16")
+    theta = jb.ParamTable([torch.empty_like(t) for t in backup.tensors], offs)
+    idx = global_index(offs, pos)
+    before = gather(backup.tensors, pos)
+    seeds = [(int(m), 9, 0) for m in synthetic.machine_ids(K, 920)]
+    q = synthetic.byte_codes(K, 920)
+    lr, denom, qs = float(F32(1e-6)), 1.0, 16.0
+    jb.jb_apply_updates_from(backup, theta, seeds, q, lr, denom, qs, write_src=write_src)
+    torch.cuda.synchronize()
+    got = gather(theta.tensors, pos)
+    src = gather(backup.tensors, pos)
+    want = oracle.update_at(before, idx, seeds, q, lr, denom, qs)
+    worst = check_theta(got, want, update_scale(before, idx, seeds, q, lr, denom, qs),
+                        f"13B update from backup K={K}")
+    assert np.array_equal(src, got if write_src else before)
+    print(f"opt-13b from backup: K={K}, {idx.size} sampled elements, worst error / allowance {worst:.3f}")
+    del backup, theta
+    free_cuda()
+
+
+def test_full_size_replay_sampled_13b(jb):
+    """A late joiner's replay (Appendix B) of 16 steps x 4 pairs on the 13B-shaped
+    bf16 set, each step rounded to storage as its own update would be: against the
+    oracle stepping the sampled elements one update at a time."""
+    table, pos, offs = _setup(jb, "opt-13b", "bf16")
+    idx = global_index(offs, pos)
+    want = gather(table.tensors, pos)
+    lr, qs = float(F32(1e-6)), 16.0
+    steps = []
+    for t in range(16):
+        seeds = [(int(m), 100 + t, 0) for m in synthetic.machine_ids(4, 930, t)]
+        steps.append((seeds, synthetic.byte_codes(4, 930, t), lr, 4.0))
+    jb.jb_replay_updates(table, [(jb.seeds_array(s), q, l, d) for s, q, l, d in steps], qs)
+    torch.cuda.synchronize()
+    got = gather(table.tensors, pos)
+    allow = np.zeros(idx.size)
+    for seeds, q, l, d in steps:
+        scale = update_scale(want, idx, seeds, q, l, d, qs)
+        allow += np.ldexp(1.0, np.frexp(scale)[1] - 8) + 2e-6 * scale
+        want = oracle.update_at(want, idx, seeds, q, l, d, qs)
+    err = np.abs(as_f64(got) - as_f64(want))
+    ratio = float((err / (allow + 1e-300)).max())
+    print(f"opt-13b replay 16 x 4: {idx.size} sampled elements, worst error / allowance {ratio:.3f}")
+    assert np.all(err <= allow + 2.0**-133), ratio
+    del table
+    free_cuda()
+
+
 def test_full_size_restore_cycle_13b(jb):
     """+eps, -2 eps, +eps on the 13B-shaped bf16 set: back within three roundings."""
     table, pos, offs = _setup(jb, "opt-13b", "bf16")
