@@ -66,10 +66,33 @@ def test_checksum_many_segments(jb):
     assert gpu_checksum(jb, table) == oracle.checksum(vals, offs)
 
 
-def test_checksum_full_size_opt13b_layout_1p3b(jb):
+def test_checksum_full_size_opt1p3b(jb):
     """The OPT-1.3B-shaped bf16 set (1.3e9 elements) against the oracle on its full copy."""
     specs, tensors, offs = synthetic.opt_parameters("opt-1.3b", torch.bfloat16)
     table = jb.ParamTable(tensors, offs)
     got = gpu_checksum(jb, table)
     host = [to_host(t) for t in tensors]
     assert got == oracle.checksum(host, offs)
+
+
+def test_checksum_full_size_opt13b(jb):
+    """The OPT-13B-shaped bf16 set (12.85e9 elements, the benchmark's launch). The
+    checksum is a sum mod 2^64 of per-window terms, and a window never spans two
+    tensors (flat offsets are multiples of 8 elements), so the whole-table value
+    must equal the sum of the 644 one-tensor values; the token embedding, 8
+    random tensors of >= 2^24 elements and random others (24 in all) are checked
+    against the oracle on their full host copies."""
+    specs, tensors, offs = synthetic.opt_parameters("opt-13b", torch.bfloat16)
+    full = gpu_checksum(jb, jb.ParamTable(tensors, offs))
+    per = [gpu_checksum(jb, jb.ParamTable([t], [fo])) for t, fo in zip(tensors, offs)]
+    assert full == sum(per) % (1 << 64)
+    rng = synthetic.rng(98)
+    big = [i for i, t in enumerate(tensors) if t.numel() >= 1 << 24]
+    picks = set(rng.choice(big, size=8, replace=False).tolist()) | {0}  # 0: the token embedding
+    picks |= set(rng.choice(len(tensors), size=24 - len(picks), replace=False).tolist())
+    for i in sorted(picks):
+        assert per[i] == oracle.checksum([to_host(tensors[i])], [offs[i]]), int(i)
+    print(f"checked against the oracle: {sum(tensors[i].numel() for i in picks)} elements "
+          f"in {len(picks)} tensors")
+    del tensors
+    torch.cuda.empty_cache()
