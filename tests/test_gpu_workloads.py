@@ -79,7 +79,11 @@ def test_full_size_perturb_sampled(jb, model, dtype, K):
     free_cuda()
 
 
-@pytest.mark.parametrize("model,dtype,K", WORKLOADS)
+# the benchmark's K sweep ends: K = 1 runs the one-pair kernel, K = 256 the seed loop
+UPDATE_WORKLOADS = WORKLOADS + [("opt-13b", "bf16", 1), ("opt-13b", "bf16", 256)]
+
+
+@pytest.mark.parametrize("model,dtype,K", UPDATE_WORKLOADS)
 def test_full_size_update_sampled(jb, model, dtype, K):
     table, pos, offs = _setup(jb, model, dtype)
     idx = global_index(offs, pos)
