@@ -12,7 +12,8 @@
  *                     (Algorithm 1, inference loop).
  *   jb_apply_updates  the step update: every machine's (seed, one-byte
  *                     projected gradient) pair applied with weight
- *                     -grad * eta / numel(all_grads) in machine-timestamp
+ *                     minus the gradient times the learning rate over the
+ *                     number of collected gradients, in machine-timestamp
  *                     order (Section 2, on applying the collected scalar projected
  *                     gradients; Algorithm 1), fused into one read and one
  *                     write of theta.
@@ -109,8 +110,8 @@ typedef struct {
     uint64_t flat_offset;
 } jb_segment;
 
-/* Seed s = (machine start-time identifier, iteration, sample index) of
- * Algorithm 1 ("s <- (self_time, t, length(projected_grads))"). 16 bytes. */
+/* Seed s of Algorithm 1: the machine's start time (as an identifier), the
+ * iteration, and the sample's index within the iteration. 16 bytes. */
 typedef struct {
     uint64_t machine_id;
     uint32_t step;
@@ -137,8 +138,9 @@ int jb_perturb(const jb_segment* segs, int n_segs, int dtype, jb_seed seed, floa
  *   c_k = (float)(-(double)lr * deq(q[k]) / (double)denom) with deq as in
  *   jb_dequantize_grad, pairs taken in ascending (machine_id, step,
  *   sample_id) order whatever order they are passed in.
- * The paper divides by numel(all_grads) (denom = K); Section 4 scales the
- * learning rate with sqrt(#perturbations): denom is therefore the caller's.
+ * The paper divides by the number of collected gradients (denom = K);
+ * Section 4 scales the learning rate with sqrt(#perturbations): denom is
+ * therefore the caller's.
  *   seeds, q, K   host arrays of K pairs (copied). K = 0 is a no-op.
  *                 K <= jb_max_seeds_per_call(); duplicates are an error.
  *   lr, denom     finite, denom != 0. qscale: S > 0 of the byte code.
@@ -150,7 +152,7 @@ int jb_apply_updates(const jb_segment* segs, int n_segs, int dtype, const jb_see
 
 /*
  * jb_apply_updates_from -- the step update applied to the weight backup, fused
- * with the restore (Algorithm 1: theta <- copy(theta_backup), then every
+ * with the restore (Algorithm 1: theta is reset from the backup copy, then every
  * machine's gradients; Section 2: the backup avoids the drift of theta + z - z):
  *   dst_e <- round_T(src_e + sum_k c_k z_e(seeds[k])), one read of src and one
  *   write of dst per element (and one more write of src when write_src != 0, so

@@ -13,7 +13,7 @@
  *   - the SPSA sample +eps, -2eps, +eps around two losses
  *                                               (Algorithm 1, inference loop)
  *   - apply every machine's projected gradients in machine-timestamp order
- *     with weight -grad * eta / numel(all_grads)
+ *     with weight minus gradient times learning rate over the number of gradients
  *                                               (Algorithm 1; Section 2)
  *   - the one-byte signed-log projected gradient clipped to +-127
  *                                               (Section 3, Training Speed)

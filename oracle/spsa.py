@@ -6,7 +6,8 @@ theta to theta_backup), so machine m evaluates its sample from the backup:
 +eps, loss, -2 eps, loss, +eps; projected gradient (l+ - l-) / (2 eps);
 one-byte code (Section 3). Then theta is restored from the backup and every
 machine's (seed, byte) pair is applied in machine-timestamp order with weight
--grad * eta / numel(all_grads) (Algorithm 1). Losses are summed in fp64.
+minus gradient times learning rate over the number of gradients (Algorithm 1).
+Losses are summed in fp64.
 """
 from __future__ import annotations
 

@@ -3,9 +3,9 @@
 // Host side of the hot path: argument checks, the canonical (machine id,
 // step, sample id) order of the pairs (Section 2: gradients are applied in
 // machine-timestamp order), the per-pair coefficients c_k = -lr deq(q_k) /
-// denom (Algorithm 1: weight -grad * eta / numel(all_grads)), the one-byte
-// code (Section 3, Training Speed), and the packing of segments and pairs
-// into kernel launches. Every element-wise step runs in the CUDA kernels.
+// denom (Algorithm 1: minus gradient times learning rate over the number of
+// gradients), the one-byte code (Section 3, Training Speed), and the packing of
+// segments and pairs into kernel launches. Every element-wise step runs in the CUDA kernels.
 #include <algorithm>
 #include <cmath>
 #include <cstring>

@@ -316,7 +316,8 @@ def test_update_k0_identity_and_k1_is_perturb():
 
 
 def test_update_coefficient_is_descent_direction():
-    """Weight -grad * eta / numel (Algorithm 1): positive gradient, negative step."""
+    """The update weight of Algorithm 1 is minus gradient times learning rate over
+    the number of gradients: a positive gradient gives a negative step."""
     with open(os.path.join(GOLDEN, "paper_constants.json")) as f:
         pc = json.load(f)
     sign = pc["update_weight"]["sign"]
