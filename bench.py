@@ -395,7 +395,7 @@ class Roofline:
       152 SMs x 128 lanes x the maximum SM clock. frac = T_roof / T_best.
     * floors.generator: the same K N element-seeds at the rate of Philox4x32-10 alone
       (jb_debug_philox_fold, measured in this run): what the wide multiplies cost.
-    * floors.mufu: one special-function operation per element-seed (rcp and rsqrt
+    * floors.mufu: one special-function operation per element-seed (rcp and sqrt
       per word pair) at 16 lanes per clock per SM.
     * issue_measured: the kernel's own ncu-measured lane-instructions per
       element-seed at peak issue (occupancy of the issue slots, not a bound)."""

@@ -35,8 +35,8 @@
  *   geometry or the GPU run, so every replica regenerates identical noise.
  *   Scope of that bit-identity: the Philox words are exact integers and the
  *   same on any machine; the transform is fp32 with every rounding explicit,
- *   except its reciprocal and reciprocal square root, which are the GPU's
- *   rcp.approx / rsqrt.approx instructions. z is therefore bitwise identical
+ *   except its reciprocal and square root, which are the GPU's
+ *   rcp.approx / sqrt.approx instructions. z is therefore bitwise identical
  *   on every sm_103a (GB300) GPU, the only target of this library; on other
  *   hardware its last bits may differ, while staying within 1e-6 of the exact
  *   definition above.

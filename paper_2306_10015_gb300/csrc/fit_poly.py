@@ -15,9 +15,10 @@ Fitted functions (the kernel's variables):
          w in [0, 16 s_max^2], s in [-1/7, 1/5] (t in [-1/4, 1/2)).
   S(y):  sin(pi x / 4) = x (pi/4 + y S(y)), y = x^2, x in [0, 1]  (first octant);
          pi/4 is applied as hi + lo so that the leading term rounds once
-  C(y):  cos(pi x / 4) = 1 + y C(y),  x in [0, 1], C of degree 2 (degree 6 in x:
-         absolute error 7.8e-8 after fp32 evaluation, within the 1e-6 budget of z
-         at the largest radius; one packed operation fewer than degree 3)
+  C(y):  cos(pi x / 4) = 1 + y C(y),  x in [0, 1], C of degree 3 (degree 8 in x;
+         degree 2 saves one packed operation but leaves an absolute error of
+         7.8e-8, too much of the 1e-6 budget of z at large radii once the radius
+         comes from sqrt.approx)
 """
 from __future__ import annotations
 
@@ -128,7 +129,7 @@ def main():
         if y == 0:
             return -(mp.pi / 4) ** 2 / 2
         return (mp.cos(mp.pi * mp.sqrt(y) / 4) - 1) / y
-    Cc = fit_rounded(C_true, [lambda y, k=k: y ** k for k in range(3)], 0, 1,
+    Cc = fit_rounded(C_true, [lambda y, k=k: y ** k for k in range(4)], 0, 1,
                      lambda y: (y + mp.mpf("1e-30")) / mp.cos(mp.pi * mp.sqrt(y) / 4))
 
     # --- measured fp32 errors of the Horner schemes ------------------------------------

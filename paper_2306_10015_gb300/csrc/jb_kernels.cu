@@ -232,34 +232,6 @@ __device__ __forceinline__ TileFast tile_fast(const P& p, uint64_t wt, uint32_t&
     return f;
 }
 
-template <typename T, int V>
-__device__ __forceinline__ void load_tile_fast(const TileFast& f, uint32_t lane, Tile<T, V>& tl) {
-    constexpr int E = Traits<T>::E;
-#pragma unroll
-    for (int j = 0; j < V; ++j) {
-        const uint32_t v = 32u * j + lane;
-        tl.blk[j] = (f.win0 + v) * (E / 4);
-        tl.full[j] = v < f.count;
-        tl.seg[j] = 0;
-        if (tl.full[j]) {
-            load_vec(reinterpret_cast<const T*>(f.base + 16ull * v), tl.x[j]);
-        } else {
-#pragma unroll
-            for (int t = 0; t < E; ++t) tl.x[j][t] = 0.0f;
-        }
-    }
-}
-
-template <typename T, int V, bool TO_DST = false>
-__device__ __forceinline__ void store_tile_fast(const TileFast& f, uint32_t lane, const Tile<T, V>& tl) {
-#pragma unroll
-    for (int j = 0; j < V; ++j) {
-        const uint32_t v = 32u * j + lane;
-        if (v < f.count)
-            store_vec(reinterpret_cast<T*>((TO_DST ? f.dst : f.base) + 16ull * v), tl.x[j]);
-    }
-}
-
 // Loads tile wt. The segment cursor s only moves forward: a thread's vector
 // indices grow from one call to the next.
 template <typename T, int V, typename P>
@@ -340,18 +312,46 @@ __device__ __forceinline__ void visit_tiles(const P& p, bool also_src, Op&& op) 
     for (uint64_t ws = warp; ws * (kTileVec * S) < n_vec; ws += n_warps) {
         const TileFast fs = tile_fast<E, V * S, sizeof(T)>(p, ws, s);
         if (fs.fast) {
-            TileFast f = fs;
+            // per-thread addresses and Philox blocks of the tile's vectors, advanced
+            // by one tile's stride per tile instead of recomputed from the tile base
+            constexpr uint64_t kStep = 16ull * kTileVec;
+            uint64_t sp[V], dp[V], bk[V];
+#pragma unroll
+            for (int j = 0; j < V; ++j) {
+                const uint64_t off = 16ull * (32u * j + lane);
+                sp[j] = fs.base + off;
+                dp[j] = fs.dst + off;
+                bk[j] = (fs.win0 + 32u * j + lane) * (E / 4);
+            }
 #pragma unroll 1
             for (uint32_t done = 0; done < fs.count; done += kTileVec) {
-                f.count = fs.count - done < kTileVec ? fs.count - done : kTileVec;
+                const uint32_t cnt = fs.count - done < kTileVec ? fs.count - done : kTileVec;
                 Tile<T, V> tl;
-                load_tile_fast<T, V>(f, lane, tl);
+#pragma unroll
+                for (int j = 0; j < V; ++j) {
+                    tl.blk[j] = bk[j];
+                    tl.full[j] = 32u * j + lane < cnt;
+                    tl.seg[j] = 0;
+                    if (tl.full[j]) {
+                        load_vec(reinterpret_cast<const T*>(sp[j]), tl.x[j]);
+                    } else {
+#pragma unroll
+                        for (int t = 0; t < E; ++t) tl.x[j][t] = 0.0f;
+                    }
+                }
                 op(tl);
-                store_tile_fast<T, V, TO_DST>(f, lane, tl);
-                if (TO_DST && also_src) store_tile_fast<T, V, false>(f, lane, tl);
-                f.base += 16ull * kTileVec;
-                f.dst += 16ull * kTileVec;
-                f.win0 += kTileVec;
+#pragma unroll
+                for (int j = 0; j < V; ++j) {
+                    if (!tl.full[j]) continue;
+                    store_vec(reinterpret_cast<T*>(TO_DST ? dp[j] : sp[j]), tl.x[j]);
+                    if (TO_DST && also_src) store_vec(reinterpret_cast<T*>(sp[j]), tl.x[j]);
+                }
+#pragma unroll
+                for (int j = 0; j < V; ++j) {
+                    sp[j] += kStep;
+                    dp[j] += kStep;
+                    bk[j] += kTileVec * (E / 4);
+                }
             }
         } else {
 #pragma unroll 1

@@ -15,13 +15,14 @@
 //           q = -4t / (2 + t) (one rcp.approx), -2 ln(1 + t) = q + q w R(w),
 //           w = q^2, R a degree-2 minimax polynomial; L = -2 e ln 2 - 2 ln(1+t)
 //           with 2 ln 2 split hi + lo (Cody & Waite 1980) so e (2 ln 2)_hi is
-//           exact; r = r0 + corr from rsqrt.approx and one Newton step,
-//           rounded once to fp32 (one fused multiply-add).
+//           exact; r = sqrt.approx(L) (relative error below 1.1e-7 over
+//           every L the transform produces; one special-function operation
+//           where rsqrt.approx and a Newton step took four packed FP ones).
 //   angle   the 24-bit angle index splits into an octant (3 bits, handled
 //           exactly by reflection, swap and sign flips) and a 21-bit offset
 //           x in (0, 1) of the octant, sin(pi x / 4) and cos(pi x / 4) by
-//           minimax polynomials of degree 7 and 6 (relative error < 0.6 ulp
-//           for the sine, also near zero; 1.0e-7 for the cosine, which the
+//           minimax polynomials of degree 7 and 8 (relative error < 0.6 ulp
+//           for the sine, also near zero; 7.2e-8 for the cosine, which the
 //           octant keeps above 0.7).
 // Coefficients: fit_poly.py (Remez exchange). The transform is checked
 // against a double-precision evaluation of the same definition over all
@@ -42,7 +43,8 @@ constexpr float kLogR0 = 0x1.5555b4p-6f, kLogR1 = 0x1.992aaap-11f, kLogR2 = 0x1.
 constexpr float kSinHi = 0x1.921fb6p-1f;   // pi/4 = hi + lo
 constexpr float kSinLo = -0x1.777a5cp-26f;
 constexpr float kSinS0 = -0x1.4abbbep-4f, kSinS1 = 0x1.465facp-9f, kSinS2 = -0x1.2db5cep-15f;
-constexpr float kCosC0 = -0x1.3bd39cp-2f, kCosC1 = 0x1.03b058p-6f, kCosC2 = -0x1.4e78bep-12f;
+constexpr float kCosC0 = -0x1.3bd3ccp-2f, kCosC1 = 0x1.03c1b0p-6f, kCosC2 = -0x1.55b2b6p-12f,
+                kCosC3 = 0x1.d4f7eep-19f;
 constexpr float kTwoLn2Hi = -0x1.62e4p+0f;       // -(2 ln 2) to 16 bits
 constexpr float kTwoLn2Lo = -0x1.7f7d1cp-19f;    // -(2 ln 2) - kTwoLn2Hi
 
@@ -128,9 +130,9 @@ __device__ __forceinline__ float rcp_approx(float x) {
     return y;
 }
 
-__device__ __forceinline__ float rsqrt_approx(float x) {
+__device__ __forceinline__ float sqrt_approx(float x) {
     float y;
-    asm("rsqrt.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    asm("sqrt.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
     return y;
 }
 
@@ -171,7 +173,7 @@ constexpr bool kPackR = JB_PACK_RADIUS, kPackA = JB_PACK_ANGLE, kPackO = JB_PACK
 // lockstep: every floating-point step is one packed fp32x2 instruction (two IEEE
 // round-to-nearest operations per issue slot), integer steps stay per pair. The
 // radius is carried with its sign flipped where a packed operation cannot negate an
-// operand (q = 4t/(2+t), L = 2 e ln 2 + 2 ln(1+t) = ln u_a^-2 negated, r0 < 0) and
+// operand (q = 4t/(2+t), L = 2 e ln 2 + 2 ln(1+t) = ln u_a^-2 negated, -r) and
 // the sign is restored in the final sign masks; round-to-nearest is odd-symmetric,
 // so no rounding differs from the unflipped formulas.
 // Polar form: rr = (-r of pair A, -r of pair B); cm, sm = the signed cosines and sines
@@ -200,11 +202,8 @@ __device__ __forceinline__ Polar2 polar2(uint4 w) {
     const float2 l_lo = fma2<kPackR>(fe, splat(-kTwoLn2Lo), lp);
     // e (2 ln 2)_hi is exact, so L is l_hi + l_lo rounded once
     const float2 L = fma2<kPackR>(fe, splat(-kTwoLn2Hi), l_lo);         // -(-2 ln u_a)
-    const float2 yr = make_float2(rsqrt_approx(-L.x), rsqrt_approx(-L.y));
-    const float2 r0 = mul2<kPackR>(L, yr);                            // -r0
-    const float2 m = fma2<kPackR>(r0, r0, L);                          // r0^2 + L
     Polar2 o;
-    o.rr = fma2<kPackR>(m, mul2<kPackR>(splat(0.5f), yr), r0); // -(r0 + corr)
+    o.rr = make_float2(-sqrt_approx(-L.x), -sqrt_approx(-L.y));       // -r
 
     // ---- angle ----
     const int32_t waA = static_cast<int32_t>(((w.y << 2) & 0xFFFFFC00u) | 0x200u);
@@ -216,7 +215,8 @@ __device__ __forceinline__ Polar2 polar2(uint4 w) {
     ps = fma2<kPackA>(y, ps, splat(kSinS0));
     ps = fma2<kPackA>(y, ps, splat(kSinLo));
     const float2 S = fma2<kPackA>(x, splat(kSinHi), mul2<kPackA>(x, ps));
-    float2 pc = fma2<kPackA>(y, splat(kCosC2), splat(kCosC1));
+    float2 pc = fma2<kPackA>(y, splat(kCosC3), splat(kCosC2));
+    pc = fma2<kPackA>(y, pc, splat(kCosC1));
     pc = fma2<kPackA>(y, pc, splat(kCosC0));
     const float2 C = fma2<kPackA>(y, pc, splat(1.0f));
     // octant bits o2 o1 o0 = word bits 31..29: |cos| and |sin| swap when o0 ^ o1;
