@@ -164,8 +164,9 @@ def test_box_muller_joint_worst(jb):
     """The radius and the angle are computed independently, so the worst |dz| pairs
     a large radius error with a large angle error. The radius of every radius word
     is read at angle word 0 (the cosine is then exactly 1, z = r); the 64 words whose
-    radius is furthest from sqrt(-2 ln u_a) in double precision are each taken with
-    all 2^24 angle words (1.07e9 draws) against the oracle."""
+    radius is furthest from sqrt(-2 ln u_a) in double precision, and the 32 largest
+    radii (where an angle error weighs most), are each taken with all 2^24 angle
+    words (1.6e9 draws) against the oracle."""
     all_a = np.arange(0, 1 << 23, dtype=np.uint32) << 9
     words = np.stack([all_a, np.zeros_like(all_a)], 1).reshape(-1)
     out = torch.empty(words.size, dtype=torch.float32, device="cuda")
@@ -174,7 +175,7 @@ def test_box_muller_joint_worst(jb):
     r_gpu = out.cpu().numpy().astype(np.float64)[0::2]
     u_a = ((all_a >> 9).astype(np.float64) + 0.5) * 2.0**-23
     dr = np.abs(r_gpu - np.sqrt(-2.0 * np.log(u_a)))
-    worst = np.argsort(dr)[-64:]
+    worst = np.union1d(np.argsort(dr)[-64:], np.arange(32))  # word 0: the largest radius
     all_b = np.arange(0, 1 << 24, dtype=np.uint32) << 8
     out = torch.empty(2 * all_b.size, dtype=torch.float32, device="cuda")
     m = 0.0
@@ -185,7 +186,7 @@ def test_box_muller_joint_worst(jb):
         sync()
         got = out.cpu().numpy().astype(np.float64).reshape(-1, 2)
         m = max(m, float(np.abs(got - oracle.box_muller_pairs(pairs)).max()))
-    print(f"largest radius error {dr.max():.3e}; max |dz| over the 64 worst radius words "
+    print(f"largest radius error {dr.max():.3e}; max |dz| over {worst.size} radius words "
           f"x every angle word: {m:.3e}")
     assert m <= Z_ABS_TOL
 
