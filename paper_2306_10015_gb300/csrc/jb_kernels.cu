@@ -413,6 +413,13 @@ __device__ __forceinline__ void accumulate_range(const P& p, const uint64_t (&bl
         uint4 w[V][B];
         tile_words<V, B>(seed_const(seed_key(p.seeds[kb])), blk, w);
         // per block: the next seed's Philox words, then this seed's transform
+        // Philox round 1's product of the block counter is the same for every seed
+        BlockCtr bc[V][B];
+#pragma unroll
+        for (int j = 0; j < V; ++j)
+#pragma unroll
+            for (int b = 0; b < B; ++b)
+                bc[j][b] = block_ctr(static_cast<uint32_t>(blk[j]) + b, static_cast<uint32_t>(blk[j] >> 32));
         for (uint32_t k = kb; k + 1 < ke; ++k) {
             const SeedConst sn = seed_const(seed_key(p.seeds[k + 1]));
             const float2 c = splat(p.seeds[k].coef);
@@ -420,8 +427,7 @@ __device__ __forceinline__ void accumulate_range(const P& p, const uint64_t (&bl
             for (int j = 0; j < V; ++j)
 #pragma unroll
                 for (int b = 0; b < B; ++b) {
-                    const uint4 wn = philox_block(sn, static_cast<uint32_t>(blk[j]) + b,
-                                                  static_cast<uint32_t>(blk[j] >> 32));
+                    const uint4 wn = philox_block(sn, bc[j][b]);
                     accum_block(w[j][b], c, acc[j][b][0], acc[j][b][1]);
                     w[j][b] = wn;
                 }
